@@ -292,3 +292,23 @@ def test_online_share_below_exact_share():
     sh = oracle.shares(a.t_ns, a.route, a.session, panel.n_labels, 32, 50_000_000)
     assert sh["A"] <= sh["P"] <= sh["U"] and sh["F"] <= sh["P"]
     assert sh["counts"]["A"] % 32 == 0
+
+
+def test_shares_do_not_depend_on_input_order():
+    panel, a = _replay(3000, horizon_s=3.0)
+    perm = np.random.default_rng(5).permutation(a.n)
+    for K in (8, 32):
+        base = _all_three(a.t_ns, a.route, panel.n_labels, K, 50_000_000)
+        shuf = _all_three(a.t_ns[perm], a.route[perm], panel.n_labels, K, 50_000_000)
+        assert base == shuf
+
+
+def test_fixed_windows_floor_toward_minus_infinity_and_follow_origin():
+    # windows [o + w*delta, o + (w+1)*delta): with origin 0 and delta 10,
+    # -5 and -1 share window -1 while 3 sits in window 0 (hand-worked)
+    t = np.array([-5, -1, 3], np.int64)
+    r = np.zeros(3, np.uint32)
+    assert oracle.fixed_count(t, r, 1, 2, 10) == 2
+    # shifting the origin to -6 puts all three in [-6, 4)
+    assert oracle.fixed_count(t, r, 1, 3, 10, origin=-6) == 3
+    assert oracle.fixed_count(t, r, 1, 3, 10, origin=0) == 0
