@@ -1,0 +1,221 @@
+/*
+ * rc.h -- C ABI of librc.so, the GB300 (sm_103a) ready-cohort transition engine.
+ *
+ * What it computes (arXiv 2608.12123, "Ready Cohorts"):
+ *   A cohort is K control events of one route, each addressed to one session.
+ *   One cohort step (Section 2.1: a transition reads typed state and an event
+ *   and emits new state, a route and possibly an effect descriptor) does, for
+ *   every member m with session s = session_idx[m] (or m), outcome o and
+ *   payload p, on that session's state record {state x, step, acc...}:
+ *     rk  = route key of (x, o, p)          (64-bit; x is the state before the step)
+ *     y   = T_sel[x][o]                     (route body sel of the two, Section 7.1)
+ *     record <- {y, step + 1, acc mixed with rk}
+ *     effect[m] = {rk, s, y | o << 16 | sel << 24}
+ *   and one global binary decision (Section 7.1: a GPU predicate computes one
+ *   global binary route decision per epoch):
+ *     d = (number of members with odd rk) > floor(K / 2)
+ *   which selects the route body of the next step.  The decision stays in the
+ *   device memory of the context; the resident mechanisms read it there and
+ *   never copy it to the host (Section 7.1, device resident path).
+ *
+ *   Exact arithmetic (the paper defines neither hash nor update; this library's
+ *   reading, identical in the separate CPU oracle):
+ *     fin(z)  = SplitMix64 output finaliser (Steele, Lea, Flood, OOPSLA 2014)
+ *     rk      = fin((x | o << 32) ^ 0x9E3779B97F4A7C15), then rk = fin(rk ^ w_k)
+ *               for each little-endian 64-bit payload word w_k in order
+ *     acc     = (acc ^ rk) * 0x9E3779B97F4A7C15                     16-byte record
+ *     acc[j]  = (acc[j] ^ rotl64(rk, 8 j)) * 0x9E3779B97F4A7C15, j<7  64-byte record
+ *   State records are little-endian: 16 bytes {int32 state, uint32 step,
+ *   uint64 acc} or 64 bytes {int32 state, uint32 step, uint64 acc[7]}.
+ *   Effects are 16 bytes {uint64 rk, uint32 session, uint32 y|o<<16|sel<<24}.
+ *
+ * Conventions for every call:
+ *   - Return RC_OK (0) or a negative RC_E_* code; rc_last_error() gives text.
+ *   - Work is asynchronous on the context's CUDA stream, except where a call
+ *     says it synchronises.  Errors that kernels find (a state >= S, an
+ *     outcome >= 8, a session index >= n_sessions, a device wait that ran out)
+ *     are latched in device memory and returned by the next synchronising call
+ *     (rc_chain and rc_sync synchronise).
+ *   - "Device pointer" means memory the GPU of the context can address
+ *     (cudaMalloc / torch CUDA tensors).  Event and output buffers may also be
+ *     host memory (pageable or pinned): the library then copies them through
+ *     its own device staging buffers on the context stream, inside the call.
+ *     The state array must be device memory.
+ *   - All buffers passed in stay owned by the caller; the library owns the
+ *     context, its device copy of the tables, the decision flag, counters,
+ *     staging buffers, pinned host words and CUDA graphs.
+ *   - Buffers must start on 16-byte boundaries.
+ *   - A context is not thread-safe: one host thread at a time.
+ */
+#ifndef RC_H
+#define RC_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define RC_OK 0
+#define RC_E_INVAL (-1)       /* bad argument; nothing launched */
+#define RC_E_CUDA (-2)        /* a CUDA runtime call failed */
+#define RC_E_DEADLINE (-3)    /* launch_ns > deadline_ns; nothing launched (Section 2.3, Eq. 1) */
+#define RC_E_STATE (-4)       /* a kernel saw state >= S or outcome >= 8 (latched) */
+#define RC_E_TIMEOUT (-5)     /* a bounded device or host wait ran out */
+#define RC_E_UNSUPPORTED (-6) /* shape or mechanism not available on this device */
+#define RC_E_INDEX (-7)       /* a kernel saw session_idx >= n_sessions (latched) */
+#define RC_E_NOMEM (-8)       /* a device or host allocation failed */
+
+typedef struct rc_ctx rc_ctx;
+
+/* How the decision of step n reaches step n + 1 (Section 7.1, Section 8.1). */
+typedef enum {
+    /* Host round trip: per step, launch the step kernel with the host's sel,
+       copy the 4-byte decision to pinned host memory, synchronise, branch on
+       the host, launch the next step. */
+    RC_MECH_HOST_RT = 0,
+    /* Device resident, CUDA-graph conditional node: one graph launch whose
+       WHILE node re-runs the step kernel; the step's last CTA sets the loop
+       handle and the flag in device memory selects the next route body. */
+    RC_MECH_RESIDENT_COND = 1,
+    /* Device resident, persistent kernel: one launch runs all steps; the
+       decision is reduced and read on device between steps (one CTA for
+       K <= 1024, a cooperative grid otherwise). */
+    RC_MECH_RESIDENT_PERSIST = 2,
+    /* Fixed nested graph (Section 8.1 negative control): per step the host
+       launches a graph whose launcher kernel device-launches a fixed child
+       graph holding the step body it chose; then the 4-byte copy, the
+       synchronisation and the host branch as in RC_MECH_HOST_RT. */
+    RC_MECH_FIXED_NESTED = 3,
+    /* No-decision floor (Section 7.1): replays a given route sequence as one
+       graph of step kernels without computing or reading any decision.  Not
+       an admissible policy; a structural floor. */
+    RC_MECH_FLOOR = 4,
+    /* The resident mechanism this build measured fastest for the shape
+       (currently the persistent kernel). */
+    RC_MECH_RESIDENT = 5
+} rc_mechanism;
+
+/* The events of one or more cohorts of K members.
+   Cohort j (0 <= j < n_sets) owns outcome[j*K .. j*K+K-1],
+   payload[(j*K) * payload_bytes ...] and session_idx[j*K ...].
+   Step n of a chain uses cohort n mod n_sets (n_sets = 0 means 1). */
+typedef struct {
+    const uint32_t *outcome;     /* outcome class per member, < 8 */
+    const uint8_t *payload;      /* payload_bytes per member */
+    const uint32_t *session_idx; /* session per member, < n_sessions, no repeats within
+                                    a cohort; NULL: member m is session m */
+    uint32_t payload_bytes;      /* must equal the context's payload_bytes */
+    uint32_t n_sets;
+    int64_t launch_ns;           /* launch time tau of the (first) cohort, integer ns */
+} rc_events;
+
+/* Creates a context.
+ *   S: number of automaton states, a power of two in [1, 256].
+ *   transition_table: HOST pointer to uint8 [2][S][8], route body A then B;
+ *     entry [b][x][o] is the next state of state x on outcome o; every entry
+ *     must be < S.  Copied to device memory.
+ *   state_bytes: 16 or 64.  payload_bytes: 32, 64 or 128.
+ *   max_K: largest cohort size the context will be given (>= 1).
+ *   n_sessions: number of records in every state array given to this context
+ *     (session indices are checked against it on the device).
+ *   cuda_stream: cudaStream_t to run on (NULL: the legacy default stream).
+ * The decision flag starts at 0 (route body A). */
+int rc_init(rc_ctx **out, uint32_t S, const uint8_t *transition_table, uint32_t state_bytes,
+            uint32_t payload_bytes, uint32_t max_K, uint64_t n_sessions, void *cuda_stream);
+
+/* One cohort step on cohort 0 of *events, with route body = the context's
+ * current decision flag; afterwards the flag holds this step's decision.
+ *   state: device pointer, n_sessions records.
+ *   K: cohort size, <= max_K (0 is allowed: nothing changes, the flag becomes 0).
+ *   deadline_ns: latest admissible launch time of the cohort (Section 2.3);
+ *     events->launch_ns > deadline_ns returns RC_E_DEADLINE and launches nothing.
+ *   effects_out: K x 16 bytes, or NULL.
+ * Asynchronous: does not synchronise. */
+int rc_cohort_step(rc_ctx *ctx, void *state, const rc_events *events, uint32_t K,
+                   int64_t deadline_ns, void *effects_out);
+
+/* A chain of n_steps cohort steps; step n uses cohort n mod events->n_sets and
+ * the route body chosen by the decision of step n - 1 (step 0: the context's
+ * current flag).  Results are identical for every admissible mechanism.
+ *   decisions_out: uint32 [n_steps], decision of each step; for RC_MECH_FLOOR
+ *     it is READ instead: it holds the route sequence to replay (step n uses
+ *     body decisions_out[n-1], step 0 the context flag).  May be NULL except
+ *     for RC_MECH_FLOOR.
+ *   effects_out: [n_steps][K] x 16 bytes, or NULL.
+ *   state_log_out: [n_steps][K] x state_bytes, the record of each member after
+ *     each step, or NULL.
+ * Synchronises before returning; returns latched device errors. */
+int rc_chain(rc_ctx *ctx, uint32_t n_steps, rc_mechanism mechanism, void *state, const rc_events *events,
+             uint32_t K, uint32_t *decisions_out, void *effects_out, void *state_log_out);
+
+/* Releases the context (synchronises its stream first).  NULL is accepted. */
+int rc_free(rc_ctx *ctx);
+
+/* Text of the last error on this context (never NULL; empty if none). */
+const char *rc_last_error(rc_ctx *ctx);
+
+/* Waits (bounded by the host wait limit) for the context stream and returns
+   any latched device error, clearing it. */
+int rc_sync(rc_ctx *ctx);
+
+/* Reads (synchronising) or sets (asynchronously) the decision flag. */
+int rc_get_decision(rc_ctx *ctx, uint32_t *sel_out);
+int rc_set_decision(rc_ctx *ctx, uint32_t sel);
+
+/* Bounds for waits: device spin waits (persistent grid barrier) give up after
+   device_ns and latch RC_E_TIMEOUT; host waits give up after host_ns. */
+int rc_set_wait_limits(rc_ctx *ctx, uint64_t device_ns, uint64_t host_ns);
+
+/* Launch-floor probes used to express small-K latency as a multiple of the
+ * platform floor.  kind: 0 = empty kernel launch + stream synchronise (host
+ * clock); 1 = empty kernel node in a graph of reps back-to-back nodes (device
+ * events); 2 = one iteration of an empty WHILE conditional graph (device
+ * events); 3 = empty kernel + 4-byte device-to-host copy + synchronise (host
+ * clock).  *us_out receives microseconds per unit. */
+int rc_launch_floor(rc_ctx *ctx, int kind, uint32_t reps, double *us_out);
+
+/* Test hook (device-side bounded-wait check): when armed, CTA 1 of the next
+   cooperative persistent launch skips its first barrier arrival, so the other
+   CTAs' bounded waits run out and RC_E_TIMEOUT is latched. */
+int rc_debug_skip_arrival(rc_ctx *ctx, uint32_t armed);
+
+/* ------------------------------------------------------------------------ */
+/* Online cohort former (host).  Section 9.1 (online runtime queueing events
+ * by route and deadline; A counts events launched by their deadline),
+ * feasibility of Eq. 1.  Events must be pushed in (t_ns, event_id) order.
+ * One open cohort per route with capacity and threshold K:
+ *   - on an arrival for route r at now = t_ns, members of r's open cohort
+ *     and of r's deferred queue with t + delta_ns < now go to fallback;
+ *   - an event whose session already sits in r's open cohort is deferred;
+ *   - the deferred queue (then the arrival) fills the open cohort in order;
+ *     at K members the cohort launches with tau = now and the queue refills
+ *     the next one.
+ * Cohorts are returned in launch order.                                      */
+typedef struct rc_former rc_former;
+
+int rc_former_create(rc_former **out, uint32_t n_routes, uint32_t K, int64_t delta_ns);
+/* Pushes one event.  Returns RC_E_INVAL on a route >= n_routes or an event
+   out of (t_ns, event_id) order. */
+int rc_former_push(rc_former *f, int64_t t_ns, uint32_t route, uint32_t session, int64_t event_id);
+/* Pops the oldest launched cohort: members_out (K event ids in cohort order),
+   *tau_out, *route_out.  Returns 1 if a cohort was popped, 0 if none is ready. */
+int rc_former_pop(rc_former *f, int64_t *members_out, int64_t *tau_out, uint32_t *route_out);
+/* Pushes n events with ids first_event_id, first_event_id + 1, ... in order;
+   stops at the first rejected event and returns its RC_E_* code. */
+int rc_former_push_many(rc_former *f, uint64_t n, const int64_t *t_ns, const uint32_t *route,
+                        const uint32_t *session, int64_t first_event_id);
+/* Pops up to max_cohorts launched cohorts into members_out [max_cohorts][K],
+   tau_out and route_out (host arrays); returns how many were popped. */
+int64_t rc_former_pop_many(rc_former *f, uint64_t max_cohorts, int64_t *members_out, int64_t *tau_out,
+                           uint32_t *route_out);
+/* Counters: events pushed, events launched, events dropped to fallback so far
+   (events still open are neither). */
+int rc_former_counts(rc_former *f, int64_t *pushed, int64_t *launched, int64_t *fallback);
+int rc_former_free(rc_former *f);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RC_H */

@@ -1,0 +1,92 @@
+// rc_internal.h -- declarations shared by the kernel and host translation units
+// of librc.so.  Not part of the public ABI (see include/rc.h).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace rc {
+
+// Library-owned device words of one context.  One 256-byte block, zeroed at
+// rc_init.  The decision flag `sel` is the HBM-resident route decision that
+// the next step reads (Section 7.1, device resident path).
+struct alignas(256) DevBlock {
+    uint32_t sel;           // route body of the next step (last decision)
+    uint32_t err;           // first latched error code (0: none)
+    uint32_t err_step;      // step of the first latched error
+    uint32_t err_member;    // member of the first latched error
+    uint32_t step;          // step counter of graph-launched chains
+    uint32_t ticket;        // last-CTA ticket of a multi-CTA step
+    uint32_t count;         // odd-key count of a multi-CTA step
+    uint32_t skip_arrival;  // test hook: CTA 1 skips its first grid-barrier arrival
+    uint32_t abort;         // set by a CTA whose bounded wait ran out
+    uint32_t pad0[3];
+    uint64_t wait_ns;       // device spin-wait limit (ns of %globaltimer)
+    unsigned long long slot[3];  // grid-barrier words of the persistent grid kernel
+    uint32_t countdown;     // launch-floor probe: WHILE iterations left
+};
+
+// Everything a step kernel needs.  Event arrays hold n_sets cohorts of K;
+// step n uses cohort n % n_sets.  Output pointers may be null.
+struct StepArgs {
+    uint8_t *state;
+    uint64_t n_sessions;
+    const uint32_t *outcome;
+    const uint8_t *payload;
+    const uint32_t *idx;
+    uint32_t n_sets;
+    uint32_t K;
+    const uint8_t *tables;   // [2][tab_stride] bytes: body A, body B
+    uint32_t S;
+    uint32_t tab_stride;     // bytes per body, a multiple of 16 (>= 8 S)
+    uint32_t *decisions;     // [n_steps]
+    uint8_t *effects;        // [n_steps][K][16]
+    uint8_t *state_log;      // [n_steps][K][state_bytes]
+    uint32_t n_steps;
+    DevBlock *dev;
+    cudaGraphConditionalHandle h_while;
+};
+
+// Epilogue flags of the per-step kernel.
+enum : uint32_t {
+    EPI_NONE = 0u,
+    EPI_SET_WHILE = 1u,  // last CTA sets the WHILE handle to (next step < n_steps)
+};
+
+// Error codes latched on the device (same values as include/rc.h).
+enum : uint32_t {
+    DEV_E_STATE = 4u,
+    DEV_E_TIMEOUT = 5u,
+    DEV_E_INDEX = 7u,
+};
+
+constexpr int kStepThreads = 256;
+constexpr int kGridThreads = 256;
+
+// Host-side launch helpers (rc_kernels.cu).
+// Per-step kernel: step < 0 reads the step from dev->step (and the last CTA
+// advances it); sel < 0 reads the route body from dev->sel.  decide = false
+// is the no-decision floor body (no reduction, flag untouched).
+const void *step_kernel(int state_bytes, int payload_bytes, bool decide);
+dim3 step_grid(uint32_t K);
+dim3 step_block(uint32_t K);
+cudaError_t launch_step(const StepArgs &a, int state_bytes, int payload_bytes, int step, int sel,
+                        uint32_t epi, bool decide, cudaStream_t s);
+
+// Persistent chains.  The single-CTA form takes K <= 1024; the grid form is a
+// cooperative launch of `grid` CTAs.
+cudaError_t launch_chain_cta(const StepArgs &a, int state_bytes, int payload_bytes, cudaStream_t s);
+cudaError_t chain_grid_size(int state_bytes, int payload_bytes, uint32_t K, int *grid);
+cudaError_t launch_chain_grid(const StepArgs &a, int state_bytes, int payload_bytes, int grid,
+                              cudaStream_t s);
+
+// Writes decisions[0..n) = 0 and sel = 0 (an empty cohort decides 0).
+cudaError_t launch_empty_cohorts(const StepArgs &a, cudaStream_t s);
+
+// Fixed-nested control: a one-thread kernel that device-launches `child`.
+const void *launcher_kernel();
+// Launch-floor probes.
+const void *empty_kernel();
+const void *countdown_kernel();
+
+}  // namespace rc

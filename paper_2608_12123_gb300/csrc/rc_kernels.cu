@@ -1,0 +1,490 @@
+// rc_kernels.cu -- sm_103a kernels of the ready-cohort transition path.
+//
+// One cohort step (Section 2.1 transition unit; Section 7.1 route bodies and
+// global binary decision) per member m, one thread per member:
+//   16-byte vector loads of the member's event (outcome, payload) and of its
+//   session's state record; route key in registers (SplitMix64 finaliser
+//   chained over the little-endian payload words); next state from the
+//   selected route body's table staged in shared memory; 16-byte vector
+//   stores of the record and the effect; odd-key count by warp ballot +
+//   popcount, per-CTA sum in shared memory, then one atomic per CTA and a
+//   last-CTA ticket (per-step kernel) or a grid barrier word (persistent).
+//
+// All work is integer; results are bit-identical to the CPU oracle.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <type_traits>
+
+#include "rc_internal.h"
+
+namespace rc {
+namespace {
+
+constexpr uint64_t kGamma = 0x9E3779B97F4A7C15ull;  // golden-ratio increment of SplitMix64
+constexpr uint64_t kFinA = 0xBF58476D1CE4E5B9ull;   // finaliser multipliers
+constexpr uint64_t kFinB = 0x94D049BB133111EBull;
+
+__device__ __forceinline__ uint64_t fin64(uint64_t z) {
+    z ^= z >> 30;
+    z *= kFinA;
+    z ^= z >> 27;
+    z *= kFinB;
+    return z ^ (z >> 31);
+}
+
+__device__ __forceinline__ uint64_t pack64(uint32_t lo, uint32_t hi) {
+    return (static_cast<uint64_t>(hi) << 32) | lo;
+}
+
+template <int R>
+__device__ __forceinline__ uint64_t rotl64c(uint64_t v) {
+    if constexpr (R % 64 == 0) {
+        return v;
+    } else {
+        return (v << (R % 64)) | (v >> (64 - R % 64));
+    }
+}
+
+// Route key: (state, outcome) packed low/high and offset by gamma, then one
+// finaliser round per 64-bit payload word.  The state is the pre-step state.
+template <int P>
+__device__ __forceinline__ uint64_t route_key(uint32_t x, uint32_t o, const uint4 (&pw)[P / 16]) {
+    uint64_t h = fin64(pack64(x, o) ^ kGamma);
+#pragma unroll
+    for (int k = 0; k < P / 16; ++k) {
+        h = fin64(h ^ pack64(pw[k].x, pw[k].y));
+        h = fin64(h ^ pack64(pw[k].z, pw[k].w));
+    }
+    return h;
+}
+
+// 64-bit word j (1..) of a record held as 16-byte vectors.
+template <int W, int NV>
+__device__ __forceinline__ uint64_t rec_word(const uint4 (&r)[NV]) {
+    return (W & 1) ? pack64(r[W / 2].z, r[W / 2].w) : pack64(r[W / 2].x, r[W / 2].y);
+}
+template <int W, int NV>
+__device__ __forceinline__ void rec_set_word(uint4 (&r)[NV], uint64_t v) {
+    if (W & 1) {
+        r[W / 2].z = static_cast<uint32_t>(v);
+        r[W / 2].w = static_cast<uint32_t>(v >> 32);
+    } else {
+        r[W / 2].x = static_cast<uint32_t>(v);
+        r[W / 2].y = static_cast<uint32_t>(v >> 32);
+    }
+}
+
+template <int J, int NV>
+__device__ __forceinline__ void mix_acc_word(uint4 (&r)[NV], uint64_t rk) {
+    rec_set_word<1 + J, NV>(r, (rec_word<1 + J, NV>(r) ^ rotl64c<8 * J>(rk)) * kGamma);
+}
+
+// acc update: one word for the 16-byte record, seven rotated words for 64.
+template <int SB>
+__device__ __forceinline__ void mix_acc(uint4 (&r)[SB / 16], uint64_t rk) {
+    constexpr int NV = SB / 16;
+    mix_acc_word<0, NV>(r, rk);
+    if constexpr (SB == 64) {
+        mix_acc_word<1, NV>(r, rk);
+        mix_acc_word<2, NV>(r, rk);
+        mix_acc_word<3, NV>(r, rk);
+        mix_acc_word<4, NV>(r, rk);
+        mix_acc_word<5, NV>(r, rk);
+        mix_acc_word<6, NV>(r, rk);
+    }
+}
+
+__device__ __forceinline__ void latch_error(DevBlock *dev, uint32_t code, uint32_t step, uint32_t member) {
+    if (atomicCAS(&dev->err, 0u, code) == 0u) {
+        dev->err_step = step;
+        dev->err_member = member;
+    }
+}
+
+__device__ __forceinline__ uint32_t ld_volatile_u32(const uint32_t *p) {
+    return *reinterpret_cast<const volatile uint32_t *>(p);
+}
+
+__device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long long *p) {
+    unsigned long long v;
+    asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void red_release_add_u64(unsigned long long *p, unsigned long long v) {
+    asm volatile("red.release.gpu.global.add.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Copies both route bodies' tables into shared memory (16-byte vectors).
+__device__ __forceinline__ void stage_tables(uint8_t *smem, const uint8_t *tables, uint32_t tab_stride,
+                                             uint32_t n_bodies, uint32_t first_body) {
+    const uint32_t nvec = tab_stride / 16 * n_bodies;
+    const uint4 *src = reinterpret_cast<const uint4 *>(tables + static_cast<size_t>(first_body) * tab_stride);
+    uint4 *dst = reinterpret_cast<uint4 *>(smem);
+    for (uint32_t i = threadIdx.x; i < nvec; i += blockDim.x) dst[i] = __ldg(src + i);
+}
+
+// The event of member m of cohort `set`.
+template <int P>
+struct Event {
+    uint32_t s;
+    uint32_t o;
+    uint4 pw[P / 16];
+};
+
+template <int P>
+__device__ __forceinline__ void load_event(Event<P> &ev, const StepArgs &a, uint32_t set, uint32_t m) {
+    const size_t e = static_cast<size_t>(set) * a.K + m;
+    ev.s = a.idx ? __ldg(a.idx + e) : m;
+    ev.o = __ldg(a.outcome + e);
+    const uint4 *p = reinterpret_cast<const uint4 *>(a.payload + e * P);
+#pragma unroll
+    for (int k = 0; k < P / 16; ++k) ev.pw[k] = __ldg(p + k);
+}
+
+// One member's transition.  Returns 1 for an odd route key, 0 for an even key
+// or a rejected member (error latched, nothing written).  `cg_state` reads the
+// state record at L2 (bypassing L1), as needed when other CTAs of a persistent
+// grid wrote it after this SM last cached it.
+template <int SB, int P, bool CG_STATE>
+__device__ __forceinline__ uint32_t transition(const StepArgs &a, const Event<P> &ev, const uint8_t *tab,
+                                               uint32_t sel, uint32_t n, uint32_t m) {
+    constexpr int NV = SB / 16;
+    if (ev.s >= a.n_sessions) {
+        latch_error(a.dev, DEV_E_INDEX, n, m);
+        return 0u;
+    }
+    uint4 *rp = reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(ev.s) * SB);
+    uint4 r[NV];
+#pragma unroll
+    for (int k = 0; k < NV; ++k) r[k] = CG_STATE ? __ldcg(rp + k) : rp[k];
+    const uint32_t x = r[0].x;
+    if (x >= a.S || ev.o >= 8u) {
+        latch_error(a.dev, DEV_E_STATE, n, m);
+        return 0u;
+    }
+    const uint64_t rk = route_key<P>(x, ev.o, ev.pw);
+    const uint32_t y = tab[x * 8u + ev.o];
+    r[0].x = y;
+    r[0].y = r[0].y + 1u;
+    mix_acc<SB>(r, rk);
+#pragma unroll
+    for (int k = 0; k < NV; ++k) rp[k] = r[k];
+    const size_t slot = static_cast<size_t>(n) * a.K + m;
+    if (a.effects) {
+        uint4 e;
+        e.x = static_cast<uint32_t>(rk);
+        e.y = static_cast<uint32_t>(rk >> 32);
+        e.z = ev.s;
+        e.w = y | (ev.o << 16) | (sel << 24);
+        __stcs(reinterpret_cast<uint4 *>(a.effects) + slot, e);
+    }
+    if (a.state_log) {
+        uint4 *lp = reinterpret_cast<uint4 *>(a.state_log + slot * SB);
+#pragma unroll
+        for (int k = 0; k < NV; ++k) __stcs(lp + k, r[k]);
+    }
+    return static_cast<uint32_t>(rk & 1u);
+}
+
+// ---------------------------------------------------------------------------
+// Per-step kernel: one launch = one cohort step (rc_cohort_step, the host
+// round trip, the graph mechanisms).
+// ---------------------------------------------------------------------------
+template <int SB, int P, bool DECIDE>
+__global__ void __launch_bounds__(kStepThreads) k_step(StepArgs a, int step_arg, int sel_arg, uint32_t epi) {
+    __shared__ __align__(16) uint8_t tab[256 * 8];
+    __shared__ uint32_t warp_odd[kStepThreads / 32];
+    __shared__ uint32_t s_step, s_sel;
+    const uint32_t tid = threadIdx.x;
+    if (tid == 0) {
+        s_step = step_arg >= 0 ? static_cast<uint32_t>(step_arg) : ld_volatile_u32(&a.dev->step);
+        s_sel = sel_arg >= 0 ? static_cast<uint32_t>(sel_arg) : (ld_volatile_u32(&a.dev->sel) & 1u);
+    }
+    __syncthreads();
+    const uint32_t n = s_step;
+    const uint32_t sel = s_sel;
+    stage_tables(tab, a.tables, a.tab_stride, 1, sel);
+    __syncthreads();
+
+    const uint32_t m = blockIdx.x * blockDim.x + tid;
+    uint32_t odd = 0;
+    if (m < a.K) {
+        Event<P> ev;
+        load_event<P>(ev, a, n % a.n_sets, m);
+        odd = transition<SB, P, false>(a, ev, tab, sel, n, m);
+    }
+    if constexpr (!DECIDE) return;
+
+    const uint32_t ball = __ballot_sync(0xffffffffu, odd);
+    if ((tid & 31u) == 0) warp_odd[tid >> 5] = __popc(ball);
+    __syncthreads();
+    if (tid != 0) return;
+    uint32_t c = 0;
+    for (uint32_t w = 0; w < (blockDim.x + 31u) / 32u; ++w) c += warp_odd[w];
+    uint32_t total = c;
+    if (gridDim.x > 1) {
+        atomicAdd(&a.dev->count, c);
+        __threadfence();
+        const uint32_t ticket = atomicAdd(&a.dev->ticket, 1u);
+        if (ticket != gridDim.x - 1) return;
+        __threadfence();
+        total = atomicExch(&a.dev->count, 0u);
+        atomicExch(&a.dev->ticket, 0u);
+    }
+    const uint32_t d = total > a.K / 2u ? 1u : 0u;
+    a.dev->sel = d;
+    if (a.decisions) a.decisions[n] = d;
+    a.dev->step = n + 1u;
+    if (epi & EPI_SET_WHILE) cudaGraphSetConditional(a.h_while, (n + 1u < a.n_steps) ? 1u : 0u);
+}
+
+// ---------------------------------------------------------------------------
+// Persistent chain, one CTA (K <= 1024): all n_steps in one launch.  The
+// decision is reduced in shared memory and read from a register: it never
+// leaves the SM.  The next step's events are fetched before the reduction.
+// ---------------------------------------------------------------------------
+template <int SB, int P>
+__global__ void __launch_bounds__(1024) k_chain_cta(StepArgs a) {
+    __shared__ __align__(16) uint8_t tab[2 * 256 * 8];
+    __shared__ uint32_t warp_odd[2][32];
+    const uint32_t tid = threadIdx.x;
+    const uint32_t nw = (blockDim.x + 31u) / 32u;
+    stage_tables(tab, a.tables, a.tab_stride, 2, 0);
+    uint32_t sel = ld_volatile_u32(&a.dev->sel) & 1u;
+    __syncthreads();
+    const bool active = tid < a.K;
+    Event<P> nxt;
+    if (active && a.n_steps > 0) load_event<P>(nxt, a, 0, tid);
+    for (uint32_t n = 0; n < a.n_steps; ++n) {
+        uint32_t odd = 0;
+        if (active) {
+            const Event<P> ev = nxt;
+            odd = transition<SB, P, false>(a, ev, tab + sel * a.tab_stride, sel, n, tid);
+            if (n + 1u < a.n_steps) load_event<P>(nxt, a, (n + 1u) % a.n_sets, tid);
+        }
+        const uint32_t ball = __ballot_sync(0xffffffffu, odd);
+        if ((tid & 31u) == 0) warp_odd[n & 1u][tid >> 5] = __popc(ball);
+        __syncthreads();  // also orders this step's state stores before the next step's loads
+        uint32_t total = 0;
+        for (uint32_t w = 0; w < nw; ++w) total += warp_odd[n & 1u][w];
+        sel = total > a.K / 2u ? 1u : 0u;
+        if (tid == 0 && a.decisions) a.decisions[n] = sel;
+    }
+    if (tid == 0) {
+        if (a.n_steps > 0) a.dev->sel = sel;
+        a.dev->step = a.n_steps;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Persistent chain, cooperative grid (any K): each CTA owns a grid-stride
+// slice of members.  Per step, thread 0 of each CTA adds (1 << 32 | odd
+// count) to the step's barrier word with release semantics and spins with
+// acquire loads until all CTAs have arrived; the low half is then the full
+// odd count, so every CTA derives the decision itself.  Three rotating words:
+// CTA 0 clears word (n+1) % 3 before arriving at step n, when no CTA can still
+// be reading it.  Spins are bounded by dev->wait_ns; on expiry the CTA latches
+// RC_E_TIMEOUT, raises dev->abort and returns, and the others follow.
+// ---------------------------------------------------------------------------
+template <int SB, int P>
+__global__ void __launch_bounds__(kGridThreads) k_chain_grid(StepArgs a) {
+    __shared__ __align__(16) uint8_t tab[2 * 256 * 8];
+    __shared__ uint32_t warp_odd[kGridThreads / 32];
+    __shared__ uint32_t s_sel, s_abort;
+    const uint32_t tid = threadIdx.x;
+    stage_tables(tab, a.tables, a.tab_stride, 2, 0);
+    if (tid == 0) {
+        s_sel = ld_volatile_u32(&a.dev->sel) & 1u;
+        s_abort = 0;
+    }
+    __syncthreads();
+    uint32_t sel = s_sel;
+    const uint32_t stride = gridDim.x * blockDim.x;
+    const uint64_t limit = a.dev->wait_ns;
+    for (uint32_t n = 0; n < a.n_steps; ++n) {
+        const uint32_t set = n % a.n_sets;
+        uint32_t odd = 0;
+        for (uint32_t m = blockIdx.x * blockDim.x + tid; m < a.K; m += stride) {
+            Event<P> ev;
+            load_event<P>(ev, a, set, m);
+            odd += transition<SB, P, true>(a, ev, tab + sel * a.tab_stride, sel, n, m);
+        }
+        // per-CTA odd count (each thread may hold more than one)
+        uint32_t v = odd;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+        if ((tid & 31u) == 0) warp_odd[tid >> 5] = v;
+        __syncthreads();
+        if (tid == 0) {
+            uint32_t c = 0;
+            for (uint32_t w = 0; w < blockDim.x / 32u; ++w) c += warp_odd[w];
+            unsigned long long *word = &a.dev->slot[n % 3u];
+            if (blockIdx.x == 0) {
+                a.dev->slot[(n + 1u) % 3u] = 0ull;
+            }
+            __threadfence();
+            const bool skip = (n == 0 && blockIdx.x == 1 && ld_volatile_u32(&a.dev->skip_arrival) != 0u);
+            if (!skip) red_release_add_u64(word, (1ull << 32) | c);
+            const uint64_t t0 = globaltimer_ns();
+            unsigned long long w;
+            uint32_t spins = 0;
+            for (;;) {
+                w = ld_acquire_u64(word);
+                if ((w >> 32) >= gridDim.x) break;
+                if ((++spins & 63u) == 0u) {
+                    if (ld_volatile_u32(&a.dev->abort) != 0u) {
+                        s_abort = 1;
+                        break;
+                    }
+                    if (globaltimer_ns() - t0 > limit) {
+                        latch_error(a.dev, DEV_E_TIMEOUT, n, blockIdx.x);
+                        atomicExch(&a.dev->abort, 1u);
+                        s_abort = 1;
+                        break;
+                    }
+                }
+            }
+            __threadfence();
+            const uint32_t d = (static_cast<uint32_t>(w & 0xffffffffull) > a.K / 2u) ? 1u : 0u;
+            s_sel = d;
+            if (blockIdx.x == 0 && a.decisions && !s_abort) a.decisions[n] = d;
+        }
+        __syncthreads();
+        if (s_abort) return;
+        sel = s_sel;
+    }
+    if (blockIdx.x == 0 && tid == 0) {
+        if (a.n_steps > 0) a.dev->sel = sel;
+        a.dev->step = a.n_steps;
+    }
+}
+
+__global__ void k_empty_cohorts(StepArgs a) {
+    for (uint32_t n = blockIdx.x * blockDim.x + threadIdx.x; n < a.n_steps; n += gridDim.x * blockDim.x)
+        if (a.decisions) a.decisions[n] = 0u;
+    if (blockIdx.x == 0 && threadIdx.x == 0 && a.n_steps > 0) {
+        a.dev->sel = 0u;
+        a.dev->step = a.n_steps;
+    }
+}
+
+// Fixed-nested control: device-launches a pre-uploaded child graph that holds
+// the route body the host chose.  It removes no host decision.
+__global__ void k_launch_child(cudaGraphExec_t child, DevBlock *dev) {
+    if (cudaGraphLaunch(child, cudaStreamGraphFireAndForget) != cudaSuccess) {
+        latch_error(dev, DEV_E_STATE, 0xffffffffu, 0xffffffffu);
+    }
+}
+
+__global__ void k_empty() {}
+
+__global__ void k_countdown(DevBlock *dev, cudaGraphConditionalHandle h) {
+    const uint32_t left = dev->countdown - 1u;
+    dev->countdown = left;
+    cudaGraphSetConditional(h, left != 0u ? 1u : 0u);
+}
+
+template <int SB, int P>
+const void *pick_step(bool decide) {
+    return decide ? reinterpret_cast<const void *>(&k_step<SB, P, true>)
+                  : reinterpret_cast<const void *>(&k_step<SB, P, false>);
+}
+
+template <int V>
+using IC = std::integral_constant<int, V>;
+
+// Calls f(IC<state_bytes>, IC<payload_bytes>) for the supported shapes.
+template <typename F>
+auto dispatch(int SB, int P, F &&f) {
+    if (SB == 16) {
+        if (P == 32) return f(IC<16>{}, IC<32>{});
+        if (P == 64) return f(IC<16>{}, IC<64>{});
+        return f(IC<16>{}, IC<128>{});
+    }
+    if (P == 32) return f(IC<64>{}, IC<32>{});
+    if (P == 64) return f(IC<64>{}, IC<64>{});
+    return f(IC<64>{}, IC<128>{});
+}
+
+}  // namespace
+
+const void *step_kernel(int SB, int P, bool decide) {
+    return dispatch(SB, P, [&](auto b, auto q) { return pick_step<decltype(b)::value, decltype(q)::value>(decide); });
+}
+
+dim3 step_block(uint32_t K) {
+    const uint32_t b = K >= static_cast<uint32_t>(kStepThreads) ? kStepThreads : ((K + 31u) / 32u) * 32u;
+    return dim3(b ? b : 32u);
+}
+
+dim3 step_grid(uint32_t K) {
+    const uint32_t b = step_block(K).x;
+    const uint32_t g = (K + b - 1u) / b;
+    return dim3(g ? g : 1u);
+}
+
+cudaError_t launch_step(const StepArgs &a, int SB, int P, int step, int sel, uint32_t epi, bool decide,
+                        cudaStream_t s) {
+    const void *fn = step_kernel(SB, P, decide);
+    StepArgs aa = a;
+    void *args[] = {&aa, &step, &sel, &epi};
+    return cudaLaunchKernel(fn, step_grid(a.K), step_block(a.K), args, 0, s);
+}
+
+cudaError_t launch_chain_cta(const StepArgs &a, int SB, int P, cudaStream_t s) {
+    const void *fn = dispatch(SB, P, [](auto b, auto q) {
+        return reinterpret_cast<const void *>(&k_chain_cta<decltype(b)::value, decltype(q)::value>);
+    });
+    StepArgs aa = a;
+    void *args[] = {&aa};
+    const uint32_t threads = ((a.K + 31u) / 32u) * 32u;
+    return cudaLaunchKernel(fn, dim3(1), dim3(threads ? threads : 32u), args, 0, s);
+}
+
+static const void *grid_fn(int SB, int P) {
+    return dispatch(SB, P, [](auto b, auto q) {
+        return reinterpret_cast<const void *>(&k_chain_grid<decltype(b)::value, decltype(q)::value>);
+    });
+}
+
+cudaError_t chain_grid_size(int SB, int P, uint32_t K, int *grid) {
+    int dev = 0, sms = 0, per_sm = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, grid_fn(SB, P), kGridThreads, 0);
+    if (e != cudaSuccess) return e;
+    const long long cap = static_cast<long long>(sms) * per_sm;
+    const long long need = (static_cast<long long>(K) + kGridThreads - 1) / kGridThreads;
+    long long g = need < cap ? need : cap;
+    if (g < 1) g = 1;
+    *grid = static_cast<int>(g);
+    return cudaSuccess;
+}
+
+cudaError_t launch_chain_grid(const StepArgs &a, int SB, int P, int grid, cudaStream_t s) {
+    StepArgs aa = a;
+    void *args[] = {&aa};
+    return cudaLaunchCooperativeKernel(grid_fn(SB, P), dim3(grid), dim3(kGridThreads), args, 0, s);
+}
+
+cudaError_t launch_empty_cohorts(const StepArgs &a, cudaStream_t s) {
+    StepArgs aa = a;
+    void *args[] = {&aa};
+    return cudaLaunchKernel(reinterpret_cast<const void *>(&k_empty_cohorts), dim3(1), dim3(256), args, 0, s);
+}
+
+const void *launcher_kernel() { return reinterpret_cast<const void *>(&k_launch_child); }
+const void *empty_kernel() { return reinterpret_cast<const void *>(&k_empty); }
+const void *countdown_kernel() { return reinterpret_cast<const void *>(&k_countdown); }
+
+}  // namespace rc

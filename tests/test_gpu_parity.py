@@ -1,0 +1,173 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle, bit
+for bit, on every decision, effect, per-step state record and final state
+(the exactness contract of Sections 2.2 and 7.3), for every mechanism of
+Section 7.1 / 8.1 and every workload shape."""
+import importlib
+
+import numpy as np
+import pytest
+
+import rc_workload as wl
+
+pytestmark = pytest.mark.gpu
+
+MECHS = ("host_rt", "resident_cond", "resident_persist", "fixed_nested", "floor")
+
+
+@pytest.fixture(scope="module")
+def g():
+    return importlib.import_module("gpu_util")
+
+
+@pytest.fixture(scope="module")
+def rc():
+    return importlib.import_module("paper_2608_12123_gb300")
+
+
+def _inputs(cfg, K, S, SB, P, n_sets, N=None):
+    tables = wl.make_tables(S, wl.stream_seed(cfg, wl.Purpose.TABLE))
+    Nn = K if N is None else N
+    state0 = wl.make_state(Nn, S, SB, wl.stream_seed(cfg, wl.Purpose.STATE))
+    outc, pay, idx = wl.make_cohort_events(cfg, n_sets, K, P, n_sessions=N)
+    return tables, state0, outc, pay, idx
+
+
+def _check_all(g, rc, mechs, tables, state0, outc, pay, idx, n_steps, K, sel0=0, log=True, what=""):
+    want = g.run_oracle(tables, state0, outc, pay, idx, n_steps, sel0=sel0, log=log)
+    for name in mechs:
+        mech = rc.MECHANISMS[name]
+        got = g.run_gpu(mech, tables, state0, outc, pay, idx, n_steps, K, sel0=sel0, log=log,
+                        floor_seq=want["decisions"])
+        w = dict(want)
+        if name == "floor":
+            w.pop("sel")  # the floor replays the sequence and leaves the flag alone
+        g.assert_same(got, w, f"{what} {name}")
+    return want
+
+
+def test_tiny_chain_all_mechanisms(g, rc):
+    # K = 32, S = 16, 16-byte records, 32-byte payloads, 1,000 chained steps
+    K, S, SB, P, n = 32, 16, 16, 32, 1000
+    tables, state0, outc, pay, idx = _inputs(1, K, S, SB, P, n)
+    want = _check_all(g, rc, MECHS, tables, state0, outc, pay, idx, n, K, what="tiny chain")
+    assert 0 < want["decisions"].sum() < n  # both route bodies are exercised
+
+
+@pytest.mark.parametrize("SB,P", [(16, 32), (16, 64), (16, 128), (64, 32), (64, 64), (64, 128)])
+@pytest.mark.parametrize("K", [1, 7, 33, 255, 257, 1000, 1025, 3001])
+def test_ragged_shapes(g, rc, SB, P, K):
+    N = 4 * K + 5
+    S = 256 if SB == 64 else 32
+    n = 6
+    tables, state0, outc, pay, idx = _inputs(40 + K % 7, K, S, SB, P, 4, N=N)
+    _check_all(g, rc, ("host_rt", "resident_cond", "resident_persist", "fixed_nested"), tables, state0, outc,
+               pay, idx, n, K, sel0=K & 1, what=f"K={K} SB={SB} P={P}")
+
+
+def test_floor_multi_cta_and_identity(g, rc):
+    K, S, SB, P, n = 700, 64, 64, 64, 12
+    tables, state0, outc, pay, idx = _inputs(7, K, S, SB, P, n)
+    _check_all(g, rc, MECHS, tables, state0, outc, pay, idx, n, K, what="identity K=700")
+
+
+def test_empty_cohort_and_zero_steps(g, rc):
+    tables, state0, outc, pay, idx = _inputs(3, 4, 16, 16, 32, 1, N=8)
+    for name in ("host_rt", "resident_persist", "resident_cond"):
+        got = g.run_gpu(rc.MECHANISMS[name], tables, state0, outc[:, :0], pay[:, :0], idx[:, :0], 5, 0, sel0=1)
+        assert np.array_equal(got["decisions"], np.zeros(5, np.uint32))
+        assert np.array_equal(got["state"], state0) and got["sel"] == 0
+        got = g.run_gpu(rc.MECHANISMS[name], tables, state0, outc, pay, idx, 0, 4, sel0=1, log=False)
+        assert np.array_equal(got["state"], state0) and got["sel"] == 1
+
+
+def test_host_buffers_give_identical_results(g, rc):
+    K, S, SB, P, n = 300, 64, 16, 64, 20
+    tables, state0, outc, pay, idx = _inputs(9, K, S, SB, P, n, N=1000)
+    want = g.run_oracle(tables, state0, outc, pay, idx, n)
+    for name in ("host_rt", "resident_persist", "resident_cond"):
+        got = g.run_gpu(rc.MECHANISMS[name], tables, state0, outc, pay, idx, n, K, host_buffers=True)
+        g.assert_same(got, want, f"host buffers {name}")
+
+
+def test_cohort_step_api_carries_the_flag_and_checks_deadlines(g, rc):
+    import torch
+    K, S, SB, P, n = 100, 32, 16, 32, 25
+    tables, state0, outc, pay, idx = _inputs(11, K, S, SB, P, n, N=400)
+    want = g.run_oracle(tables, state0, outc, pay, idx, n)
+    ctx = rc.rc_init(S, tables, SB, P, K, 400, torch.cuda.current_stream())
+    try:
+        state = g.dev(state0.copy())
+        for j in range(n):
+            ev = rc.make_events(g.dev(outc[j]), g.dev(pay[j]), g.dev(idx[j]), n_sets=1, launch_ns=1000 + j)
+            eff = torch.zeros(K * 16, dtype=torch.uint8, device="cuda")
+            if j == 3:
+                with pytest.raises(rc.RcError) as e:
+                    rc.rc_cohort_step(ctx, state, ev, K, 1000 + j - 1, eff)
+                assert e.value.code == rc.RC_E_DEADLINE
+            rc.rc_cohort_step(ctx, state, ev, K, 1000 + j, eff)
+            assert np.array_equal(g.host(eff, np.uint8).reshape(K, 16), want["effects"][j])
+            assert rc.rc_get_decision(ctx) == want["decisions"][j]
+        rc.rc_sync(ctx)
+        assert np.array_equal(g.host(state, np.uint8).reshape(state0.shape), want["state"])
+    finally:
+        rc.rc_free(ctx)
+
+
+def test_bad_inputs_are_latched_and_the_context_survives(g, rc):
+    import torch
+    K, S, SB, P, n = 64, 16, 16, 32, 3
+    tables, state0, outc, pay, idx = _inputs(13, K, S, SB, P, n, N=200)
+    cases = []
+    o2 = outc.copy(); o2[1, 5] = 8
+    cases.append(("outcome", state0, o2, idx, rc.RC_E_STATE))
+    s2 = state0.copy(); s2[idx[0, 9], 0:4] = np.frombuffer(np.uint32(S).tobytes(), np.uint8)
+    cases.append(("state", s2, outc, idx, rc.RC_E_STATE))
+    i2 = idx.copy(); i2[2, 17] = 200
+    cases.append(("index", state0, outc, i2, rc.RC_E_INDEX))
+    for name in ("host_rt", "resident_persist", "resident_cond", "fixed_nested"):
+        for what, st, oc, ix, code in cases:
+            with pytest.raises(rc.RcError) as e:
+                g.run_gpu(rc.MECHANISMS[name], tables, st, oc, pay, ix, n, K)
+            assert e.value.code == code, (name, what)
+    # the device stays usable: a clean chain right after matches the oracle
+    want = g.run_oracle(tables, state0, outc, pay, idx, n)
+    g.assert_same(g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K), want, "after errors")
+
+
+def test_grid_barrier_wait_is_bounded(g, rc):
+    """A CTA that never arrives (test hook) makes the others' bounded waits run
+    out: RC_E_TIMEOUT comes back and the context keeps working."""
+    import torch
+    K, S, SB, P, n = 4096, 16, 16, 32, 4
+    tables, state0, outc, pay, idx = _inputs(17, K, S, SB, P, 2, N=5000)
+    ctx = rc.rc_init(S, tables, SB, P, K, 5000, torch.cuda.current_stream())
+    try:
+        rc.rc_set_wait_limits(ctx, 2_000_000, 30_000_000_000)  # 2 ms device waits
+        state = g.dev(state0.copy())
+        ev = rc.make_events(g.dev(outc), g.dev(pay), g.dev(idx))
+        dec = torch.zeros(n, dtype=torch.int32, device="cuda")
+        rc.rc_debug_skip_arrival(ctx, True)
+        with pytest.raises(rc.RcError) as e:
+            rc.rc_chain(ctx, n, rc.RC_MECH_RESIDENT_PERSIST, state, ev, K, dec)
+        assert e.value.code == rc.RC_E_TIMEOUT
+        # hook disarmed: the same context runs a clean chain
+        state = g.dev(state0.copy())
+        rc.rc_set_decision(ctx, 0)
+        rc.rc_chain(ctx, n, rc.RC_MECH_RESIDENT_PERSIST, state, ev, K, dec)
+        want = g.run_oracle(tables, state0, outc, pay, idx, n, log=False)
+        assert np.array_equal(g.host(dec, np.uint32), want["decisions"])
+        assert np.array_equal(g.host(state, np.uint8).reshape(state0.shape), want["state"])
+    finally:
+        rc.rc_free(ctx)
+
+
+def test_launch_floor_probes_run(g, rc):
+    import torch
+    tables, state0, *_ = _inputs(1, 32, 16, 16, 32, 1)
+    ctx = rc.rc_init(16, tables, 16, 32, 32, 32, torch.cuda.current_stream())
+    try:
+        for kind in (0, 1, 2, 3):
+            us = rc.rc_launch_floor(ctx, kind, 200)
+            assert 0.0 < us < 1000.0
+    finally:
+        rc.rc_free(ctx)
