@@ -1,0 +1,508 @@
+#!/usr/bin/env python3
+"""Benchmark of the ready-cohort transition path on GB300.
+
+Headline workload (one step = one device-resident chain over 1,000 formed
+cohorts of the primary cohort replay): synthetic stationary Poisson arrivals
+for 100,000 target active sessions over 60 s, K = 256, launch deadline 50 ms,
+S = 64 states, 16-byte state records, 64-byte payloads; cohorts come from the
+library's online former.  Reported: microseconds per invocation (= one cohort
+step) for the device-resident path and for the host round trip, the CUDA-graph
+and fixed-nested controls and the no-decision floor; transitions/s; the
+32-step horizon the paper reports; the launch floor; the large-K bandwidth
+case (1,048,576 sessions, K = 65,536, 64-byte records, 128-byte payloads,
+S = 256) against the measured HBM peak; end-to-end time through the C ABI
+with pinned host buffers; and the CPU oracle as a baseline.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+Multi-GPU: the path does not shard (one global decision per step), so N > 1
+runs N independent replicas under torchrun; the line reports whole-job values.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import rc_workload as wl  # noqa: E402
+
+H = 1000                   # cohort steps (invocations) per bench step
+C2 = wl.CONFIGS[2]
+C4 = wl.CONFIGS[4]
+BYTES_PER_TRANSITION_C2 = 16 + 16 + 4 + 64 + 16 + 4     # state r/w, outcome, payload, effect, index
+BYTES_PER_TRANSITION_C4 = 64 + 64 + 4 + 128 + 16 + 4
+METRIC = "us/invocation at K=256, device-resident (vs host round trip); transitions/s; HBM GB/s"
+UNIT = "us/invocation"
+WORKLOAD = ("primary cohort replay: Poisson arrivals for C=100,000 active sessions over 60 s, K=256, "
+            "deadline 50 ms, S=64, 16-byte state, 64-byte payload; 1,000 formed cohorts per step")
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=30)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", default="native", choices=["native", "reference"])
+    p.add_argument("--skip-large-k", action="store_true", help="omit the large-K bandwidth section")
+    p.add_argument("--skip-cpu", action="store_true", help="omit the CPU-oracle baseline leg")
+    p.add_argument("--large-k-only", action="store_true", help="run only the large-K section (profiling)")
+    p.add_argument("--large-k-steps", type=int, default=1000)
+    p.add_argument("--only-resident", action="store_true",
+                   help="time only the resident chain of the headline workload (profiling)")
+    p.add_argument("--no-flush", action="store_true", help="do not allocate or write the L2 flush buffer (profiling)")
+    return p.parse_args()
+
+
+# ---------------------------------------------------------------------------
+# workload set-up
+# ---------------------------------------------------------------------------
+
+def make_config2(use_oracle_former=False):
+    panel = wl.make_panel()
+    arr = wl.make_arrivals(C2["C"], panel, horizon_s=C2["horizon_s"])
+    if use_oracle_former:
+        import oracle
+        members, tau, croute = oracle.former(arr.t_ns, arr.route, arr.session, panel.n_labels, C2["K"],
+                                             C2["delta_ns"])
+    else:
+        import paper_2608_12123_gb300 as rc
+        members, tau, croute = rc.form_cohorts(arr.t_ns, arr.route, arr.session, panel.n_labels, C2["K"],
+                                               C2["delta_ns"])
+    K, P, S = C2["K"], C2["payload_bytes"], C2["S"]
+    outcome = (arr.route[members] % 8).astype(np.uint32)
+    idx = arr.session[members].astype(np.uint32)
+    payload = wl.payload_for_events(members.reshape(-1), P).reshape(len(members), K, P)
+    tables = wl.make_tables(S, wl.stream_seed(2, wl.Purpose.TABLE))
+    state0 = wl.make_state(arr.n_sessions, S, C2["state_bytes"], wl.stream_seed(2, wl.Purpose.STATE))
+    return dict(panel=panel, arr=arr, members=members, tau=tau, outcome=outcome, idx=idx, payload=payload,
+                tables=tables, state0=state0, n_cohorts=len(members))
+
+
+def make_config4(n_sets):
+    K, P, S, N = C4["K"], C4["payload_bytes"], C4["S"], C4["N"]
+    tables = wl.make_tables(S, wl.stream_seed(4, wl.Purpose.TABLE))
+    state0 = wl.make_state(N, S, C4["state_bytes"], wl.stream_seed(4, wl.Purpose.STATE))
+    outc, pay, idx = wl.make_cohort_events(4, n_sets, K, P, n_sessions=N)
+    return dict(tables=tables, state0=state0, outcome=outc, payload=pay, idx=idx)
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+
+class Clocks:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.lines = []
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [ln for ln in out.splitlines() if ln.strip()]
+        return False
+
+    def summary(self):
+        sm, mx, pw, reasons = [], [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for ln in getattr(self, "lines", []):
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+                pw.append(float(f[3]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "power_w_max": max(pw),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# helpers
+# ---------------------------------------------------------------------------
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}, "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    for name in ("rc_kernels.cu", "rc_internal.h"):
+        with open(os.path.join(ROOT, "paper_2608_12123_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic(kernel_key, units_per_launch):
+    """DRAM bytes per launch of a kernel from the committed ncu summary, scaled
+    to this launch's units, or None when the kernel changed since the capture."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            t = json.load(f)
+    except OSError:
+        return None
+    ent = t.get(kernel_key)
+    if not ent or ent.get("source_hash") != kernel_source_hash():
+        return None
+    return ent["dram_bytes_per_unit"] * units_per_launch
+
+
+def flush_l2(buf):
+    if buf is not None:
+        buf.zero_()
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+# ---------------------------------------------------------------------------
+# the native arm
+# ---------------------------------------------------------------------------
+
+def chain_on_window(rc, ctx, mech, state, dev_ev, start, n, K, dec, eff, seq=None):
+    o, p, i = dev_ev
+    ev = rc.make_events(o[start:start + n], p[start:start + n], i[start:start + n], payload_bytes=p.shape[-1],
+                        n_sets=n)
+    if mech == rc.RC_MECH_FLOOR:
+        rc.rc_chain(ctx, n, mech, state, ev, K, seq, eff, None)
+    else:
+        rc.rc_chain(ctx, n, mech, state, ev, K, dec, eff, None)
+    return rc.rc_last_chain_stats(ctx)
+
+
+def native(args):
+    import torch
+    import paper_2608_12123_gb300 as rc
+
+    world, rank, local = dist_env()
+    torch.cuda.set_device(local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    peaks, peak_src = measured_peaks()
+    hbm_peak = float(peaks["hbm_gbs"])
+    out = {}
+    K = C2["K"]
+    stream = torch.cuda.current_stream()
+    flush = None if args.no_flush else torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device="cuda")
+
+    if not args.large_k_only:
+        w = make_config2()
+        nc = w["n_cohorts"]
+        S, SB, P = C2["S"], C2["state_bytes"], C2["payload_bytes"]
+        ctx = rc.rc_init(S, w["tables"], SB, P, K, w["arr"].n_sessions, stream)
+        state = torch.from_numpy(w["state0"].copy()).cuda()
+        dev_ev = (torch.from_numpy(w["outcome"].view(np.int32)).cuda(), torch.from_numpy(w["payload"]).cuda(),
+                  torch.from_numpy(w["idx"].view(np.int32)).cuda())
+        dec = torch.zeros(H, dtype=torch.int32, device="cuda")
+        eff = torch.empty(H * K * 16, dtype=torch.uint8, device="cuda")
+        n_windows = nc // H
+        windows = [(j % n_windows) * H for j in range(args.warmup + args.steps)]
+
+        def timed(mech, steps, warm, seq=None):
+            dev_ms, launches = [], 0
+            for j in range(warm + steps):
+                flush_l2(flush)
+                ms, nl = chain_on_window(rc, ctx, mech, state, dev_ev, windows[j % len(windows)], H, K, dec, eff,
+                                         seq)
+                if j >= warm:
+                    dev_ms.append(ms)
+                    launches += nl
+            return dev_ms, launches
+
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize()
+        with Clocks(local) as clk:
+            t_wall0 = time.perf_counter()
+            res_ms, launches = timed(rc.RC_MECH_RESIDENT_PERSIST, args.steps, args.warmup)
+            torch.cuda.synchronize()
+            t_wall = time.perf_counter() - t_wall0
+            seq = np.ascontiguousarray(dec.cpu().numpy().view(np.uint32))
+            if args.only_resident:
+                rc.rc_free(ctx)
+                print(json.dumps({"resident_us_per_invocation": float(np.mean(res_ms)) * 1000.0 / H,
+                                  "gpu_launches": launches}))
+                return None
+            host_ms, _ = timed(rc.RC_MECH_HOST_RT, max(3, args.steps // 3), 2)
+            cond_ms, _ = timed(rc.RC_MECH_RESIDENT_COND, max(3, args.steps // 3), 2)
+            nest_ms, _ = timed(rc.RC_MECH_FIXED_NESTED, max(3, args.steps // 3), 2)
+            floor_ms, _ = timed(rc.RC_MECH_FLOOR, max(3, args.steps // 3), 2, seq=seq)
+        torch.cuda.synchronize()
+        step_ms = float(np.mean(res_ms))
+        if world > 1:
+            t = torch.tensor([step_ms], device="cuda")
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+            step_ms = float(t.item())
+        us_inv = step_ms * 1000.0 / H
+        value = us_inv / world  # whole job: all ranks' invocations in the slowest rank's time
+        mech_us = {name: float(np.median(v)) * 1000.0 / H for name, v in
+                   (("resident_persist", res_ms), ("host_rt", host_ms), ("resident_cond", cond_ms),
+                    ("fixed_nested", nest_ms), ("floor", floor_ms))}
+
+        # the paper's unit: one 32-step horizon per call (resident vs host round trip)
+        def horizon(mech, reps=200):
+            tot = []
+            for j in range(reps + 5):
+                ms, _ = chain_on_window(rc, ctx, mech, state, dev_ev, (j * 32) % (nc - 32), 32, K, dec, eff)
+                if j >= 5:
+                    tot.append(ms * 1000.0)
+            return float(np.median(tot))
+        hz = {"resident_persist": horizon(rc.RC_MECH_RESIDENT_PERSIST), "host_rt": horizon(rc.RC_MECH_HOST_RT),
+              "resident_cond": horizon(rc.RC_MECH_RESIDENT_COND)}
+        floor_probe = {name: rc.rc_launch_floor(ctx, kind, 2000 if kind in (0, 3) else 1000) for name, kind in
+                       (("launch_sync", 0), ("graph_node", 1), ("while_iteration", 2), ("launch_d2h_sync", 3))}
+
+        # end to end through the C ABI: events from pinned host memory, decisions
+        # and effects back to pinned host memory, inside the timed region
+        ho = torch.from_numpy(w["outcome"].view(np.int32)).pin_memory()
+        hp = torch.from_numpy(w["payload"]).pin_memory()
+        hi = torch.from_numpy(w["idx"].view(np.int32)).pin_memory()
+        hdec = torch.zeros(H, dtype=torch.int32).pin_memory()
+        heff = torch.empty(H * K * 16, dtype=torch.uint8).pin_memory()
+        e2e_s = []
+        for j in range(args.warmup + args.steps):
+            s0 = windows[j % len(windows)]
+            ev = rc.make_events(ho[s0:s0 + H], hp[s0:s0 + H], hi[s0:s0 + H], payload_bytes=P, n_sets=H)
+            flush_l2(flush)
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            rc.rc_chain(ctx, H, rc.RC_MECH_RESIDENT, state, ev, K, hdec, heff, None)
+            t1 = time.perf_counter()
+            if j >= args.warmup:
+                e2e_s.append(t1 - t0)
+        e2e_us = float(np.mean(e2e_s)) * 1e6 / H / world
+        h2d = H * K * (4 + P + 4)
+        d2h = H * 4 + H * K * 16
+
+        alg_bytes = H * K * BYTES_PER_TRANSITION_C2
+        ach = alg_bytes / (step_ms * 1e-3) / 1e9
+        traffic = ncu_traffic("k_chain_cta<16,64>", H * K)
+        out.update({
+            "metric": METRIC, "value": round(value, 4), "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(step_ms, 4), "higher_is_better": False,
+            "scaling": "weak", "vs_baseline": None, "dtype": "u64",
+            "data": "synthetic (seeded SplitMix64 Poisson replay; the paper's trace panel is not available)",
+            "config": {"workload": WORKLOAD, "K": K, "S": S, "state_bytes": SB, "payload_bytes": P,
+                       "invocations_per_step": H, "formed_cohorts": nc, "sessions": w["arr"].n_sessions,
+                       "events": w["arr"].n, "mechanism": "resident_persist (one persistent CTA)",
+                       "l2": "flushed between timed steps (512 MiB write)",
+                       "parallelism": "replicas" if world > 1 else "single GPU"},
+            "host_rt_us_per_invocation": round(mech_us["host_rt"] / world, 4),
+            "ratio_host_rt_over_resident": round(mech_us["host_rt"] / mech_us["resident_persist"], 3),
+            "mechanisms_us_per_invocation": {k: round(v, 4) for k, v in mech_us.items()},
+            "transitions_per_s": round(world * H * K / (step_ms * 1e-3), 1),
+            "horizon32_us": {k: round(v, 2) for k, v in hz.items()},
+            "launch_floor_us": {k: round(v, 3) for k, v in floor_probe.items()},
+            "latency_x_floor": {"vs_graph_node": round(us_inv / floor_probe["graph_node"], 3),
+                                "vs_while_iteration": round(us_inv / floor_probe["while_iteration"], 3),
+                                "vs_launch_sync": round(us_inv / floor_probe["launch_sync"], 3)},
+            "roofline": {"bound": "hbm", "achieved": round(ach, 3), "peak": hbm_peak, "unit": "GB/s",
+                         "frac": round(ach / hbm_peak, 5), "traffic": traffic,
+                         "kernel": "k_chain_cta<16,64> (one launch = 1,000 steps x 256 members)",
+                         "peak_source": f"{peak_src} hbm_gbs",
+                         "note": "K=256 steps are latency-bound: see latency_x_floor"},
+            "e2e": {"value": round(e2e_us, 4), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "gpu_launches": launches,
+            "clocks": clk.summary(),
+            "context": {"paper_per_epoch_us": {"resident": [8.1, 9.7], "host_rt": [14.6, 19.5]},
+                        "paper_horizon32_us_at_N256": {"resident": [258.3, 309.0], "host_rt": [467.2, 625.3]},
+                        "paper_placements": "local GTX 1660 Ti, Modal L4, RunPod L4, Lambda H100 SXM5",
+                        "paper_row_median_ratio_range": [1.19, 2.39]},
+            "timed_wall_s": round(t_wall, 3),
+        })
+        rc.rc_free(ctx)
+        del state, dev_ev, dec, eff
+
+    if not args.skip_large_k:
+        out["large_k"] = large_k(args, rc, torch, stream, hbm_peak, peak_src, flush, world)
+        if args.large_k_only:
+            print(json.dumps(out["large_k"]))
+            return None
+        out["roofline_large_k"] = out["large_k"].pop("roofline")
+    out["tiny_chain"] = tiny_chain(rc, torch, stream)
+
+    if rank == 0 and world == 1 and not args.skip_cpu:
+        out["cpu_baseline"] = cpu_baseline(w, seq_check=True)
+    return out if rank == 0 else None
+
+
+def large_k(args, rc, torch, stream, hbm_peak, peak_src, flush, world):
+    """1,048,576 sessions with 64-byte records, K = 65,536 per invocation,
+    128-byte payloads, S = 256; 1,000 invocations per chain over a ring of 64
+    event sets (about 550 MB, larger than L2)."""
+    n_sets = C4["n_sets"]
+    w = make_config4(n_sets)
+    K, S, SB, P, N = C4["K"], C4["S"], C4["state_bytes"], C4["payload_bytes"], C4["N"]
+    n = args.large_k_steps
+    ctx = rc.rc_init(S, w["tables"], SB, P, K, N, stream)
+    state = torch.from_numpy(w["state0"]).cuda()
+    o = torch.from_numpy(w["outcome"].view(np.int32)).cuda()
+    p = torch.from_numpy(w["payload"]).cuda()
+    i = torch.from_numpy(w["idx"].view(np.int32)).cuda()
+    ev = rc.make_events(o, p, i, payload_bytes=P, n_sets=n_sets)
+    dec = torch.zeros(n, dtype=torch.int32, device="cuda")
+    eff = torch.empty(n * K * 16, dtype=torch.uint8, device="cuda")
+    res = {}
+    for name, mech, reps in (("resident_persist", rc.RC_MECH_RESIDENT_PERSIST, 4),
+                             ("resident_cond", rc.RC_MECH_RESIDENT_COND, 2),
+                             ("host_rt", rc.RC_MECH_HOST_RT, 2)):
+        ms_l = []
+        for r in range(reps + 1):
+            flush_l2(flush)
+            rc.rc_chain(ctx, n, mech, state, ev, K, dec, eff, None)
+            ms, _ = rc.rc_last_chain_stats(ctx)
+            if r > 0:
+                ms_l.append(ms)
+        res[name] = float(np.median(ms_l))
+    rc.rc_free(ctx)
+    ms = res["resident_persist"]
+    us_inv = ms * 1000.0 / n
+    alg = BYTES_PER_TRANSITION_C4 * K
+    gbs = alg * n / (ms * 1e-3) / 1e9
+    return {
+        "workload": "bandwidth-bound large cohort: N=1,048,576 sessions, 64-byte state, K=65,536 sampled "
+                    "without replacement, 128-byte payload, S=256, 1,000 invocations over 64 event sets",
+        "us_per_invocation": {k: round(v * 1000.0 / n, 4) for k, v in res.items()},
+        "ratio_host_rt_over_resident": round(res["host_rt"] / ms, 3),
+        "transitions_per_s": round(world * K * n / (ms * 1e-3), 1),
+        "hbm_gbs": round(gbs, 1),
+        "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": hbm_peak, "unit": "GB/s",
+                     "frac": round(gbs / hbm_peak, 4), "traffic": ncu_traffic("k_chain_grid<64,128>", K),
+                     "kernel": "k_chain_grid<64,128> per invocation (cooperative persistent grid)",
+                     "algorithmic_bytes_per_invocation": alg, "peak_source": f"{peak_src} hbm_gbs (burst)"},
+        "l2": "inputs larger than L2 (64 MiB state + 550 MB event ring + 1 GiB effects) and flushed per chain",
+        "us_per_invocation_resident": round(us_inv, 4),
+    }
+
+
+def tiny_chain(rc, torch, stream):
+    """K = 32, S = 16, 16-byte records, 32-byte payloads, 1,000 chained steps,
+    device-resident only: latency per step as a multiple of the launch floor."""
+    c = wl.CONFIGS[1]
+    K, S, SB, P, n = c["K"], c["S"], c["state_bytes"], c["payload_bytes"], c["n_steps"]
+    tables = wl.make_tables(S, wl.stream_seed(1, wl.Purpose.TABLE))
+    state0 = wl.make_state(K, S, SB, wl.stream_seed(1, wl.Purpose.STATE))
+    outc, pay, _ = wl.make_cohort_events(1, n, K, P)
+    ctx = rc.rc_init(S, tables, SB, P, K, K, stream)
+    state = torch.from_numpy(state0).cuda()
+    ev = rc.make_events(torch.from_numpy(outc.view(np.int32)).cuda(), torch.from_numpy(pay).cuda())
+    dec = torch.zeros(n, dtype=torch.int32, device="cuda")
+    out = {}
+    for name, mech in (("resident_persist", rc.RC_MECH_RESIDENT_PERSIST), ("resident_cond", rc.RC_MECH_RESIDENT_COND),
+                       ("host_rt", rc.RC_MECH_HOST_RT)):
+        l = []
+        for r in range(6):
+            rc.rc_chain(ctx, n, mech, state, ev, K, dec, None, None)
+            if r:
+                l.append(rc.rc_last_chain_stats(ctx)[0])
+        out[name] = round(float(np.median(l)) * 1000.0 / n, 4)
+    fl = rc.rc_launch_floor(ctx, 1, 1000)
+    rc.rc_free(ctx)
+    return {"workload": "tiny chain: K=32, S=16, 16-byte state, 32-byte payload, 1,000 steps",
+            "us_per_step": out, "x_graph_node_floor": round(out["resident_persist"] / fl, 3)}
+
+
+def cpu_baseline(w, seq_check=False, n_cohorts=None):
+    """The CPU oracle as it stands (single thread) on a bounded sample: the
+    first cohorts of the same formed sequence."""
+    import oracle
+    K = C2["K"]
+    n = n_cohorts or w["n_cohorts"]
+    st = w["state0"].copy()
+    t0 = time.perf_counter()
+    r = oracle.chain(w["tables"], st, w["outcome"][:n], w["payload"][:n], w["idx"][:n], n, log=False)
+    dt = time.perf_counter() - t0
+    return {"value": round(dt * 1e6 / n, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"oracle chain over the first {n} formed cohorts of the workload ({n * K} transitions)",
+            "transitions_per_s": round(n * K / dt, 1), "seconds": round(dt, 3),
+            "decisions_digest": hashlib.sha256(r["decisions"].tobytes()).hexdigest()[:16]}
+
+
+# ---------------------------------------------------------------------------
+# the reference arm: the CPU oracle, timed as it stands
+# ---------------------------------------------------------------------------
+
+def reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return None
+    import oracle
+    w = make_config2(use_oracle_former=True)
+    K = C2["K"]
+    n = H  # cohorts per step, as in the native arm
+    times = []
+    st = w["state0"].copy()
+    for j in range(args.warmup + args.steps):
+        s0 = (j * n) % (w["n_cohorts"] - n)
+        t0 = time.perf_counter()
+        oracle.chain(w["tables"], st, w["outcome"][s0:s0 + n], w["payload"][s0:s0 + n], w["idx"][s0:s0 + n], n,
+                     log=False)
+        if j >= args.warmup:
+            times.append(time.perf_counter() - t0)
+    us = float(np.mean(times)) * 1e6 / n
+    return {"impl": "reference", "metric": METRIC, "value": round(us, 4), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(float(np.mean(times)) * 1e3, 4),
+            "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "u64",
+            "data": "synthetic", "config": {"workload": WORKLOAD, "K": K,
+                                             "invocations_per_step": n, "parallelism": "single CPU thread"},
+            "cpu_baseline": {"value": round(us, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
+                             "sample": f"{n} formed cohorts per step ({n * K} transitions)"},
+            "e2e": {"value": round(us, 4), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    args = parse_args()
+    out = reference(args) if args.impl == "reference" else native(args)
+    if out is not None:
+        print(json.dumps(out))
+
+
+if __name__ == "__main__":
+    main()

@@ -175,6 +175,13 @@ int rc_set_wait_limits(rc_ctx *ctx, uint64_t device_ns, uint64_t host_ns);
  * clock).  *us_out receives microseconds per unit. */
 int rc_launch_floor(rc_ctx *ctx, int kind, uint32_t reps, double *us_out);
 
+/* Device time of the last rc_chain's mechanism work, from CUDA events the
+   library records on the context stream just before the first and just after
+   the last operation of the mechanism (staging copies excluded), and the
+   number of executions of this library's kernels that work caused (host or
+   graph launched). */
+int rc_last_chain_stats(rc_ctx *ctx, double *device_ms_out, uint32_t *kernel_launches_out);
+
 /* Test hook (device-side bounded-wait check): when armed, CTA 1 of the next
    cooperative persistent launch skips its first barrier arrival, so the other
    CTAs' bounded waits run out and RC_E_TIMEOUT is latched. */

@@ -42,7 +42,7 @@ MECHANISMS = {"host_rt": RC_MECH_HOST_RT, "resident_cond": RC_MECH_RESIDENT_COND
 #: every symbol include/rc.h declares
 EXPORTS = ("rc_init", "rc_cohort_step", "rc_chain", "rc_free", "rc_last_error", "rc_sync",
            "rc_get_decision", "rc_set_decision", "rc_set_wait_limits", "rc_launch_floor",
-           "rc_debug_skip_arrival", "rc_former_create", "rc_former_push", "rc_former_pop",
+           "rc_debug_skip_arrival", "rc_last_chain_stats", "rc_former_create", "rc_former_push", "rc_former_pop",
            "rc_former_push_many", "rc_former_pop_many", "rc_former_counts", "rc_former_free")
 
 
@@ -70,6 +70,7 @@ def _load():
         "rc_set_wait_limits": (i, [vp, u64, u64]),
         "rc_launch_floor": (i, [vp, i, u32, P(C.c_double)]),
         "rc_debug_skip_arrival": (i, [vp, u32]),
+        "rc_last_chain_stats": (i, [vp, P(C.c_double), P(u32)]),
         "rc_former_create": (i, [P(vp), u32, u32, i64]),
         "rc_former_push": (i, [vp, i64, u32, u32, i64]),
         "rc_former_pop": (i, [vp, vp, P(i64), P(u32)]),
@@ -202,6 +203,14 @@ def rc_launch_floor(ctx, kind, reps) -> float:
     v = C.c_double()
     _check(ctx, _lib.rc_launch_floor(ctx.handle, kind, reps, C.byref(v)))
     return float(v.value)
+
+
+def rc_last_chain_stats(ctx):
+    """(device milliseconds, kernel launches) of the last rc_chain's mechanism work."""
+    ms = C.c_double()
+    n = C.c_uint32()
+    _check(ctx, _lib.rc_last_chain_stats(ctx.handle, C.byref(ms), C.byref(n)))
+    return float(ms.value), int(n.value)
 
 
 def rc_debug_skip_arrival(ctx, armed=True):

@@ -9,6 +9,7 @@
 #include <chrono>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <string>
 #include <vector>
@@ -83,6 +84,10 @@ struct rc_ctx {
     Buf st_outcome, st_payload, st_idx, st_dec, st_eff, st_log;
     CachedGraph cond, floor;
     NestedGraphs nested;
+    cudaEvent_t ev_start = nullptr, ev_stop = nullptr;
+    double last_ms = 0.0;
+    uint32_t last_launches = 0;
+    bool no_tma = false;  // RC_NO_TMA=1 in the environment selects the plain grid kernel
 };
 
 namespace {
@@ -369,11 +374,18 @@ int run_persist(rc_ctx *c, const rc::StepArgs &a) {
         return RC_OK;
     }
     if (!c->coop) return fail(c, RC_E_UNSUPPORTED, "device lacks cooperative launch");
-    int grid = 0;
-    RC_CUDA(c, rc::chain_grid_size(c->SB, c->P, a.K, &grid));
     RC_CUDA(c, cudaMemsetAsync(c->dev->slot, 0, sizeof(c->dev->slot), c->stream));
     RC_CUDA(c, cudaMemsetAsync(&c->dev->abort, 0, sizeof(uint32_t), c->stream));
-    RC_CUDA(c, rc::launch_chain_grid(a, c->SB, c->P, grid, c->stream));
+    int grid = 0;
+    uint32_t threads = 0;
+    size_t smem = 0;
+    alignas(8) unsigned char shape[32];
+    if (!c->no_tma && rc::chain_grid_tma_plan(c->SB, c->P, a.K, c->tab_stride, &grid, &threads, &smem, shape)) {
+        RC_CUDA(c, rc::launch_chain_grid_tma(a, c->SB, c->P, grid, threads, smem, shape, c->stream));
+    } else {
+        RC_CUDA(c, rc::chain_grid_size(c->SB, c->P, a.K, &grid));
+        RC_CUDA(c, rc::launch_chain_grid(a, c->SB, c->P, grid, c->stream));
+    }
     // the test hook arms one launch only
     RC_CUDA(c, cudaMemsetAsync(&c->dev->skip_arrival, 0, sizeof(uint32_t), c->stream));
     return RC_OK;
@@ -488,6 +500,10 @@ int rc_init(rc_ctx **out, uint32_t S, const uint8_t *table, uint32_t state_bytes
     c->n_sessions = n_sessions;
     c->tab_stride = ((S * 8u + 15u) / 16u) * 16u;
     c->stream = static_cast<cudaStream_t>(cuda_stream);
+    {
+        const char *v = std::getenv("RC_NO_TMA");
+        c->no_tma = v && v[0] == '1';
+    }
     auto bail = [&](cudaError_t e) {
         rc_free(c);
         (void)e;
@@ -511,6 +527,8 @@ int rc_init(rc_ctx **out, uint32_t S, const uint8_t *table, uint32_t state_bytes
     if ((e = cudaMemcpy(c->dev, &init, sizeof(init), cudaMemcpyHostToDevice)) != cudaSuccess) return bail(e);
     if ((e = cudaHostAlloc(reinterpret_cast<void **>(&c->h_pinned), 64, cudaHostAllocDefault)) != cudaSuccess)
         return bail(e);
+    if ((e = cudaEventCreate(&c->ev_start)) != cudaSuccess) return bail(e);
+    if ((e = cudaEventCreate(&c->ev_stop)) != cudaSuccess) return bail(e);
     std::memset(c->h_pinned, 0, 64);
     *out = c;
     return RC_OK;
@@ -550,10 +568,19 @@ int rc_chain(rc_ctx *c, uint32_t n_steps, rc_mechanism mech, void *state, const 
     int rc = resolve(c, state, ev, K, n_steps, decisions, effects, state_log, floor, &r);
     if (rc != RC_OK) return rc;
     if (floor) r.a.decisions = nullptr;
+    c->last_ms = 0.0;
+    c->last_launches = 0;
     if (n_steps == 0) return finish(c);
+    RC_CUDA(c, cudaEventRecord(c->ev_start, c->stream));
     if (K == 0) {
         if (!floor) RC_CUDA(c, rc::launch_empty_cohorts(r.a, c->stream));
+        c->last_launches = floor ? 0u : 1u;
     } else {
+        // kernel executions: one per step, two per step for the nested control
+        // (launcher + child), one for the persistent kernel
+        c->last_launches = mech == RC_MECH_RESIDENT_PERSIST ? 1u
+                           : mech == RC_MECH_FIXED_NESTED  ? 2u * n_steps
+                                                           : n_steps;
         switch (mech) {
             case RC_MECH_HOST_RT: rc = run_host_rt(c, r.a); break;
             case RC_MECH_RESIDENT_COND: rc = run_cond(c, r.a); break;
@@ -564,9 +591,13 @@ int rc_chain(rc_ctx *c, uint32_t n_steps, rc_mechanism mech, void *state, const 
         }
         if (rc != RC_OK) return rc;
     }
+    RC_CUDA(c, cudaEventRecord(c->ev_stop, c->stream));
     rc = copy_back(c, r, n_steps);
     if (rc != RC_OK) return rc;
-    return finish(c);
+    rc = finish(c);
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, c->ev_start, c->ev_stop) == cudaSuccess) c->last_ms = ms;
+    return rc;
 }
 
 int rc_free(rc_ctx *c) {
@@ -580,6 +611,8 @@ int rc_free(rc_ctx *c) {
     if (c->d_tables) cudaFree(c->d_tables);
     if (c->dev) cudaFree(c->dev);
     if (c->h_pinned) cudaFreeHost(c->h_pinned);
+    if (c->ev_start) cudaEventDestroy(c->ev_start);
+    if (c->ev_stop) cudaEventDestroy(c->ev_stop);
     delete c;
     return RC_OK;
 }
@@ -612,6 +645,13 @@ int rc_set_wait_limits(rc_ctx *c, uint64_t device_ns, uint64_t host_ns) {
     c->dev_wait_ns = device_ns;
     c->host_wait_ns = host_ns;
     RC_CUDA(c, cudaMemcpy(&c->dev->wait_ns, &device_ns, sizeof(uint64_t), cudaMemcpyHostToDevice));
+    return RC_OK;
+}
+
+int rc_last_chain_stats(rc_ctx *c, double *device_ms_out, uint32_t *kernel_launches_out) {
+    if (!c) return RC_E_INVAL;
+    if (device_ms_out) *device_ms_out = c->last_ms;
+    if (kernel_launches_out) *kernel_launches_out = c->last_launches;
     return RC_OK;
 }
 

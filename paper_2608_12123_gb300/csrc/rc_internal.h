@@ -80,6 +80,13 @@ cudaError_t chain_grid_size(int state_bytes, int payload_bytes, uint32_t K, int 
 cudaError_t launch_chain_grid(const StepArgs &a, int state_bytes, int payload_bytes, int grid,
                               cudaStream_t s);
 
+// TMA-fed persistent grid (K a multiple of 8, one CTA per SM).  plan returns
+// false when it does not apply; shape_out points to 32 bytes of opaque shape.
+bool chain_grid_tma_plan(int state_bytes, int payload_bytes, uint32_t K, uint32_t tab_stride, int *grid,
+                         uint32_t *threads, size_t *smem, void *shape_out);
+cudaError_t launch_chain_grid_tma(const StepArgs &a, int state_bytes, int payload_bytes, int grid, uint32_t threads,
+                                  size_t smem, const void *shape, cudaStream_t s);
+
 // Writes decisions[0..n) = 0 and sel = 0 (an empty cohort decides 0).
 cudaError_t launch_empty_cohorts(const StepArgs &a, cudaStream_t s);
 

@@ -11,6 +11,7 @@
 //   last-CTA ticket (per-step kernel) or a grid barrier word (persistent).
 //
 // All work is integer; results are bit-identical to the CPU oracle.
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -120,6 +121,61 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
     uint64_t t;
     asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
     return t;
+}
+
+// ---- shared-memory barriers and bulk / tensor copies (sm_90+ PTX) ----------
+__device__ __forceinline__ uint32_t smem_addr(const void *p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count) : "memory");
+}
+
+// One arrival that also announces `bytes` of asynchronous copies.
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
+    uint32_t done;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(smem_addr(bar)), "r"(parity)
+        : "memory");
+    return done != 0u;
+}
+
+// 2-D tiled tensor load (box of the map) into shared memory, completing on bar.
+__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, int32_t x, int32_t y, uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+            smem_addr(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
+        : "memory");
+}
+
+// Contiguous bulk copy global -> shared (16-byte aligned, size a multiple of 16).
+__device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     smem_addr(dst)),
+                 "l"(src), "r"(bytes), "r"(smem_addr(bar))
+                 : "memory");
+}
+
+// Orders this thread's earlier generic-proxy shared accesses before later
+// async-proxy (TMA) accesses of the same shared memory.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Makes mbarrier initialisation visible to the async proxy.
+__device__ __forceinline__ void fence_mbar_init() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
 }
 
 // Copies both route bodies' tables into shared memory (16-byte vectors).
@@ -367,6 +423,189 @@ __global__ void __launch_bounds__(kGridThreads) k_chain_grid(StepArgs a) {
     }
 }
 
+// ---------------------------------------------------------------------------
+// Persistent chain, cooperative grid, TMA-fed (K a multiple of 8; one CTA per
+// SM).  CTA b owns the contiguous members [b*chunk, b*chunk + cnt).  Each step
+// its events arrive in shared memory ahead of time: the payload rows as
+// n_boxes tiles of box_rows x P bytes through a 2-D tensor map whose 32/64/128
+// byte swizzle makes the per-member row reads bank-conflict free, the outcome
+// and session-index runs as 1-D bulk copies; all complete on one mbarrier per
+// stage.  Two stages: the copies for step n + 2 are issued right after the CTA
+// arrives at the grid barrier of step n, so they stream while the barrier
+// resolves.  The state gather stays after the barrier (records written by
+// other CTAs in step n must be visible).  The barrier and the decision are
+// those of k_chain_grid.  Every wait is bounded; a CTA that gives up waits
+// (bounded) for its own copies in flight before it returns.
+// ---------------------------------------------------------------------------
+struct TmaShape {
+    uint32_t chunk;        // members per CTA (multiple of 8)
+    uint32_t box_rows;     // rows per tensor tile (multiple of 8, <= 256)
+    uint32_t n_boxes;      // tiles per stage
+    uint32_t stage_pay;    // payload bytes per stage (multiple of 1024)
+    uint32_t stage_words;  // 32-bit words per outcome / index stage (multiple of 4)
+};
+
+template <int P>
+__device__ __forceinline__ void read_payload_swizzled(uint4 (&pw)[P / 16], const uint8_t *stage, uint32_t row) {
+    // TMA swizzle: 16-byte chunk bits [4..] of the shared address XOR address
+    // bits [7..] (3 bits for 128-byte rows, 2 for 64, 1 for 32); stages are
+    // 1024-byte aligned, so offsets stand for addresses.
+    constexpr uint32_t mask = P == 128 ? 7u : (P == 64 ? 3u : 1u);
+#pragma unroll
+    for (int k = 0; k < P / 16; ++k) {
+        uint32_t off = row * P + static_cast<uint32_t>(k) * 16u;
+        off ^= ((off >> 7) & mask) << 4;
+        pw[k] = *reinterpret_cast<const uint4 *>(stage + off);
+    }
+}
+
+template <int SB, int P>
+__global__ void __launch_bounds__(512, 1)
+    k_chain_grid_tma(const __grid_constant__ CUtensorMap tmap, StepArgs a, TmaShape sh) {
+    extern __shared__ uint8_t dsm_raw[];
+    __shared__ __align__(8) uint64_t bar[2];
+    __shared__ uint32_t warp_odd[16];
+    __shared__ uint32_t s_sel, s_abort, s_pending, s_pend_step[2];
+    // carve the dynamic shared memory: [pay 0][pay 1][out 0][out 1][idx 0][idx 1][tables]
+    const uint32_t raw = smem_addr(dsm_raw);
+    uint8_t *const base = dsm_raw + (((raw + 1023u) & ~1023u) - raw);
+    uint32_t *const words = reinterpret_cast<uint32_t *>(base + 2 * sh.stage_pay);
+    uint8_t *const tab = reinterpret_cast<uint8_t *>(words + 4 * sh.stage_words);
+    auto pay_of = [&](uint32_t st) { return base + st * sh.stage_pay; };
+    auto out_of = [&](uint32_t st) { return words + st * sh.stage_words; };
+    auto idx_of = [&](uint32_t st) { return words + (2u + st) * sh.stage_words; };
+
+    const uint32_t tid = threadIdx.x;
+    const uint32_t m0 = blockIdx.x * sh.chunk;
+    const uint32_t cnt = m0 < a.K ? min(sh.chunk, a.K - m0) : 0u;
+    const uint64_t limit = a.dev->wait_ns;
+
+    // thread 0 issues the copies of step j into stage j & 1
+    auto issue = [&](uint32_t j) {
+        const uint32_t st = j & 1u;
+        const uint32_t row0 = (j % a.n_sets) * a.K + m0;
+        const uint32_t bytes = sh.n_boxes * sh.box_rows * P + cnt * 4u * (a.idx ? 2u : 1u);
+        mbar_arrive_expect_tx(&bar[st], bytes);
+        for (uint32_t b = 0; b < sh.n_boxes; ++b)
+            tma_load_2d(pay_of(st) + b * sh.box_rows * P, &tmap, 0, static_cast<int32_t>(row0 + b * sh.box_rows),
+                        &bar[st]);
+        bulk_load(out_of(st), a.outcome + row0, cnt * 4u, &bar[st]);
+        if (a.idx) bulk_load(idx_of(st), a.idx + row0, cnt * 4u, &bar[st]);
+        s_pending |= 1u << st;
+        s_pend_step[st] = j;
+    };
+    // bounded wait for stage st's copies; false when it gave up
+    auto wait_stage = [&](uint32_t st, uint32_t parity) -> bool {
+        const uint64_t t0 = globaltimer_ns();
+        uint32_t spins = 0;
+        while (!mbar_try_wait(&bar[st], parity)) {
+            if ((++spins & 255u) == 0u && globaltimer_ns() - t0 > limit) return false;
+        }
+        return true;
+    };
+
+    if (tid == 0) {
+        mbar_init(&bar[0], 1);
+        mbar_init(&bar[1], 1);
+        fence_mbar_init();
+        s_sel = ld_volatile_u32(&a.dev->sel) & 1u;
+        s_abort = 0;
+        s_pending = 0;
+    }
+    stage_tables(tab, a.tables, a.tab_stride, 2, 0);
+    __syncthreads();
+    if (tid == 0 && cnt > 0) {
+        if (a.n_steps > 0) issue(0);
+        if (a.n_steps > 1) issue(1);
+    }
+    uint32_t sel = s_sel;
+    for (uint32_t n = 0; n < a.n_steps; ++n) {
+        const uint32_t st = n & 1u;
+        uint32_t odd = 0;
+        if (cnt > 0) {
+            if (!wait_stage(st, (n >> 1) & 1u)) {
+                latch_error(a.dev, DEV_E_TIMEOUT, n, blockIdx.x);
+                atomicExch(&a.dev->abort, 1u);
+                s_abort = 1;
+            }
+        }
+        __syncthreads();
+        if (s_abort) break;
+        for (uint32_t t = tid; t < cnt; t += blockDim.x) {
+            Event<P> ev;
+            ev.s = a.idx ? idx_of(st)[t] : m0 + t;
+            ev.o = out_of(st)[t];
+            read_payload_swizzled<P>(ev.pw, pay_of(st), t);
+            odd += transition<SB, P, true>(a, ev, tab + sel * a.tab_stride, sel, n, m0 + t);
+        }
+        uint32_t v = odd;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+        if ((tid & 31u) == 0) warp_odd[tid >> 5] = v;
+        __syncthreads();  // every thread is done with stage st and has stored this step's records
+        if (tid == 0) {
+            if (cnt > 0) s_pending &= ~(1u << st);
+            uint32_t c = 0;
+            for (uint32_t w = 0; w < (blockDim.x + 31u) / 32u; ++w) c += warp_odd[w];
+            unsigned long long *word = &a.dev->slot[n % 3u];
+            if (blockIdx.x == 0) a.dev->slot[(n + 1u) % 3u] = 0ull;
+            __threadfence();
+            const bool skip = (n == 0 && blockIdx.x == 1 && ld_volatile_u32(&a.dev->skip_arrival) != 0u);
+            if (!skip) red_release_add_u64(word, (1ull << 32) | c);
+            if (cnt > 0 && n + 2u < a.n_steps) {
+                fence_proxy_async_smem();
+                issue(n + 2u);
+            }
+            const uint64_t t0 = globaltimer_ns();
+            unsigned long long w;
+            uint32_t spins = 0;
+            for (;;) {
+                w = ld_acquire_u64(word);
+                if ((w >> 32) >= gridDim.x) break;
+                if ((++spins & 63u) == 0u) {
+                    if (ld_volatile_u32(&a.dev->abort) != 0u) {
+                        s_abort = 1;
+                        break;
+                    }
+                    if (globaltimer_ns() - t0 > limit) {
+                        latch_error(a.dev, DEV_E_TIMEOUT, n, blockIdx.x);
+                        atomicExch(&a.dev->abort, 1u);
+                        s_abort = 1;
+                        break;
+                    }
+                }
+            }
+            __threadfence();
+            const uint32_t d = (static_cast<uint32_t>(w & 0xffffffffull) > a.K / 2u) ? 1u : 0u;
+            s_sel = d;
+            if (blockIdx.x == 0 && a.decisions && !s_abort) a.decisions[n] = d;
+        }
+        __syncthreads();
+        if (s_abort) break;
+        sel = s_sel;
+    }
+    if (s_abort) {
+        // drain this CTA's copies still in flight (bounded) before leaving
+        if (tid == 0) {
+            for (uint32_t st = 0; st < 2; ++st) {
+                if (!(s_pending & (1u << st))) continue;
+                // the pending use of stage st is step s_pend_step[st]: its phase parity
+                const uint32_t parity = (s_pend_step[st] >> 1) & 1u;
+                const uint64_t t0 = globaltimer_ns();
+                while (!mbar_try_wait(&bar[st], parity)) {
+                    if (globaltimer_ns() - t0 > limit) break;
+                }
+            }
+        }
+        __syncthreads();
+        return;
+    }
+    if (blockIdx.x == 0 && tid == 0) {
+        if (a.n_steps > 0) a.dev->sel = sel;
+        a.dev->step = a.n_steps;
+    }
+}
+
 __global__ void k_empty_cohorts(StepArgs a) {
     for (uint32_t n = blockIdx.x * blockDim.x + threadIdx.x; n < a.n_steps; n += gridDim.x * blockDim.x)
         if (a.decisions) a.decisions[n] = 0u;
@@ -475,6 +714,96 @@ cudaError_t launch_chain_grid(const StepArgs &a, int SB, int P, int grid, cudaSt
     StepArgs aa = a;
     void *args[] = {&aa};
     return cudaLaunchCooperativeKernel(grid_fn(SB, P), dim3(grid), dim3(kGridThreads), args, 0, s);
+}
+
+static const void *grid_tma_fn(int SB, int P) {
+    return dispatch(SB, P, [](auto b, auto q) {
+        return reinterpret_cast<const void *>(&k_chain_grid_tma<decltype(b)::value, decltype(q)::value>);
+    });
+}
+
+namespace {
+using EncodeTiled = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                 const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                 CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiled encode_fn() {
+    static EncodeTiled fn = nullptr;
+    if (!fn) {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiled>(p);
+    }
+    return fn;
+}
+
+size_t tma_smem_bytes(const TmaShape &sh, uint32_t tab_stride) {
+    return 1024 + 2ull * sh.stage_pay + 4ull * sh.stage_words * 4 + 2ull * tab_stride;
+}
+}  // namespace
+
+// Chooses the TMA grid shape for K members, or returns false when the TMA
+// kernel does not apply (K not a multiple of 8, or a stage would not fit).
+bool chain_grid_tma_plan(int SB, int P, uint32_t K, uint32_t tab_stride, int *grid, uint32_t *threads,
+                         size_t *smem, void *shape_out) {
+    if (K == 0 || K % 8u != 0u || !encode_fn()) return false;
+    int dev = 0, sms = 0, max_optin = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return false;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return false;
+    if (cudaDeviceGetAttribute(&max_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+        return false;
+    TmaShape sh;
+    uint32_t per = (K + static_cast<uint32_t>(sms) - 1u) / static_cast<uint32_t>(sms);
+    sh.chunk = (per + 7u) & ~7u;
+    const uint32_t g = (K + sh.chunk - 1u) / sh.chunk;
+    sh.n_boxes = (sh.chunk + 255u) / 256u;
+    sh.box_rows = (((sh.chunk + sh.n_boxes - 1u) / sh.n_boxes) + 7u) & ~7u;
+    sh.stage_pay = ((sh.n_boxes * sh.box_rows * static_cast<uint32_t>(P)) + 1023u) & ~1023u;
+    sh.stage_words = (sh.chunk + 3u) & ~3u;
+    const size_t bytes = tma_smem_bytes(sh, tab_stride);
+    if (bytes + 2048 > static_cast<size_t>(max_optin)) return false;
+    const void *fn = grid_tma_fn(SB, P);
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes)) !=
+        cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    const uint32_t thr = sh.chunk >= 512u ? 512u : ((sh.chunk + 31u) / 32u) * 32u;
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, static_cast<int>(thr), bytes) != cudaSuccess ||
+        per_sm < 1 || static_cast<long long>(per_sm) * sms < g)
+        return false;
+    *grid = static_cast<int>(g);
+    *threads = thr;
+    *smem = bytes;
+    *static_cast<TmaShape *>(shape_out) = sh;
+    return true;
+}
+
+cudaError_t launch_chain_grid_tma(const StepArgs &a, int SB, int P, int grid, uint32_t threads, size_t smem,
+                                  const void *shape, cudaStream_t s) {
+    const TmaShape &sh = *static_cast<const TmaShape *>(shape);
+    EncodeTiled enc = encode_fn();
+    if (!enc) return cudaErrorNotSupported;
+    alignas(64) CUtensorMap map;
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(P), static_cast<cuuint64_t>(a.n_sets) * a.K};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(P)};
+    const cuuint32_t box[2] = {static_cast<cuuint32_t>(P), sh.box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUtensorMapSwizzle swz = P == 128 ? CU_TENSOR_MAP_SWIZZLE_128B
+                                   : P == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                             : CU_TENSOR_MAP_SWIZZLE_32B;
+    CUresult r = enc(&map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t *>(a.payload), dims, strides, box,
+                     estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    StepArgs aa = a;
+    TmaShape shc = sh;
+    void *args[] = {&map, &aa, &shc};
+    return cudaLaunchCooperativeKernel(grid_tma_fn(SB, P), dim3(grid), dim3(threads), args, smem, s);
 }
 
 cudaError_t launch_empty_cohorts(const StepArgs &a, cudaStream_t s) {

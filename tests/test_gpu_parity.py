@@ -171,3 +171,45 @@ def test_launch_floor_probes_run(g, rc):
             assert 0.0 < us < 1000.0
     finally:
         rc.rc_free(ctx)
+
+
+@pytest.mark.parametrize("tma", [True, False])
+@pytest.mark.parametrize("SB,P", [(16, 32), (16, 64), (64, 128), (64, 32)])
+@pytest.mark.parametrize("K,N,identity", [(1032, 5000, False), (4104, 9001, False), (2048, 2048, True),
+                                          (65536, 70000, False)])
+def test_persistent_grid_kernels(g, rc, monkeypatch, tma, SB, P, K, N, identity):
+    """The cooperative persistent kernels: the TMA-fed one (K a multiple of 8)
+    and the plain one, on member counts that do not split evenly over SMs."""
+    monkeypatch.setenv("RC_NO_TMA", "0" if tma else "1")
+    S = 256 if SB == 64 else 64
+    tables, state0, outc, pay, idx = _inputs(50 + K % 11, K, S, SB, P, 3, N=None if identity else N)
+    n = 5
+    want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=1)
+    got = g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K, sel0=1)
+    g.assert_same(got, want, f"grid tma={tma} K={K} SB={SB} P={P}")
+
+
+@pytest.mark.parametrize("tma", [True, False])
+def test_grid_barrier_wait_is_bounded_both_kernels(g, rc, monkeypatch, tma):
+    import torch
+    monkeypatch.setenv("RC_NO_TMA", "0" if tma else "1")
+    K, S, SB, P, n = 8192, 16, 16, 64, 4
+    tables, state0, outc, pay, idx = _inputs(19, K, S, SB, P, 2, N=9000)
+    ctx = rc.rc_init(S, tables, SB, P, K, 9000, torch.cuda.current_stream())
+    try:
+        rc.rc_set_wait_limits(ctx, 2_000_000, 30_000_000_000)
+        state = g.dev(state0.copy())
+        ev = rc.make_events(g.dev(outc), g.dev(pay), g.dev(idx))
+        dec = torch.zeros(n, dtype=torch.int32, device="cuda")
+        rc.rc_debug_skip_arrival(ctx, True)
+        with pytest.raises(rc.RcError) as e:
+            rc.rc_chain(ctx, n, rc.RC_MECH_RESIDENT_PERSIST, state, ev, K, dec)
+        assert e.value.code == rc.RC_E_TIMEOUT
+        state = g.dev(state0.copy())
+        rc.rc_set_decision(ctx, 0)
+        rc.rc_chain(ctx, n, rc.RC_MECH_RESIDENT_PERSIST, state, ev, K, dec)
+        want = g.run_oracle(tables, state0, outc, pay, idx, n, log=False)
+        assert np.array_equal(g.host(dec, np.uint32), want["decisions"])
+        assert np.array_equal(g.host(state, np.uint8).reshape(state0.shape), want["state"])
+    finally:
+        rc.rc_free(ctx)
