@@ -42,7 +42,7 @@ MECHANISMS = {"host_rt": RC_MECH_HOST_RT, "resident_cond": RC_MECH_RESIDENT_COND
 #: every symbol include/rc.h declares
 EXPORTS = ("rc_init", "rc_cohort_step", "rc_chain", "rc_free", "rc_last_error", "rc_sync",
            "rc_get_decision", "rc_set_decision", "rc_set_wait_limits", "rc_launch_floor",
-           "rc_debug_skip_arrival", "rc_last_chain_stats", "rc_former_create", "rc_former_push", "rc_former_pop",
+           "rc_debug_skip_arrival", "rc_last_chain_stats", "rc_set_trace", "rc_former_create", "rc_former_push", "rc_former_pop",
            "rc_former_push_many", "rc_former_pop_many", "rc_former_counts", "rc_former_free")
 
 
@@ -71,6 +71,7 @@ def _load():
         "rc_launch_floor": (i, [vp, i, u32, P(C.c_double)]),
         "rc_debug_skip_arrival": (i, [vp, u32]),
         "rc_last_chain_stats": (i, [vp, P(C.c_double), P(u32)]),
+        "rc_set_trace": (i, [vp, vp, u64]),
         "rc_former_create": (i, [P(vp), u32, u32, i64]),
         "rc_former_push": (i, [vp, i64, u32, u32, i64]),
         "rc_former_pop": (i, [vp, vp, P(i64), P(u32)]),
@@ -211,6 +212,15 @@ def rc_last_chain_stats(ctx):
     n = C.c_uint32()
     _check(ctx, _lib.rc_last_chain_stats(ctx.handle, C.byref(ms), C.byref(n)))
     return float(ms.value), int(n.value)
+
+
+def rc_set_trace(ctx, buf, nbytes=None):
+    """Points the profiling trace at a device buffer (None turns it off)."""
+    if buf is None:
+        return _check(ctx, _lib.rc_set_trace(ctx.handle, None, 0))
+    if nbytes is None:
+        nbytes = buf.numel() * buf.element_size()
+    return _check(ctx, _lib.rc_set_trace(ctx.handle, _ptr(buf), int(nbytes)))
 
 
 def rc_debug_skip_arrival(ctx, armed=True):

@@ -87,7 +87,10 @@ struct rc_ctx {
     cudaEvent_t ev_start = nullptr, ev_stop = nullptr;
     double last_ms = 0.0;
     uint32_t last_launches = 0;
-    bool no_tma = false;  // RC_NO_TMA=1 in the environment selects the plain grid kernel
+    bool no_tma = false;   // RC_NO_TMA=1 in the environment selects the plain grid kernel
+    bool no_pipe = false;  // RC_NO_PIPE=1 selects the plain single-CTA kernel
+    long long *trace = nullptr;
+    uint64_t trace_entries = 0;
 };
 
 namespace {
@@ -220,6 +223,7 @@ int resolve(rc_ctx *c, void *state, const rc_events *ev, uint32_t K, uint32_t n_
     a.n_steps = n_steps;
     a.dev = c->dev;
     a.h_while = 0;
+    a.trace = (c->trace && c->trace_entries >= 12ull * n_steps) ? c->trace : nullptr;
     const size_t n_ev = static_cast<size_t>(n_sets) * K;
     a.outcome = ev->outcome;
     a.payload = ev->payload;
@@ -370,7 +374,9 @@ int run_cond(rc_ctx *c, const rc::StepArgs &a) {
 // ---- device resident: persistent kernel ------------------------------------
 int run_persist(rc_ctx *c, const rc::StepArgs &a) {
     if (a.K <= 1024u) {
-        RC_CUDA(c, rc::launch_chain_cta(a, c->SB, c->P, c->stream));
+        bool launched = false;
+        if (!c->no_pipe) RC_CUDA(c, rc::launch_chain_cta_fast(a, c->SB, c->P, c->stream, &launched));
+        if (!launched) RC_CUDA(c, rc::launch_chain_cta(a, c->SB, c->P, c->stream));
         return RC_OK;
     }
     if (!c->coop) return fail(c, RC_E_UNSUPPORTED, "device lacks cooperative launch");
@@ -503,6 +509,8 @@ int rc_init(rc_ctx **out, uint32_t S, const uint8_t *table, uint32_t state_bytes
     {
         const char *v = std::getenv("RC_NO_TMA");
         c->no_tma = v && v[0] == '1';
+        const char *w = std::getenv("RC_NO_PIPE");
+        c->no_pipe = w && w[0] == '1';
     }
     auto bail = [&](cudaError_t e) {
         rc_free(c);
@@ -652,6 +660,15 @@ int rc_last_chain_stats(rc_ctx *c, double *device_ms_out, uint32_t *kernel_launc
     if (!c) return RC_E_INVAL;
     if (device_ms_out) *device_ms_out = c->last_ms;
     if (kernel_launches_out) *kernel_launches_out = c->last_launches;
+    return RC_OK;
+}
+
+int rc_set_trace(rc_ctx *c, void *device_buf, uint64_t bytes) {
+    if (!c) return RC_E_INVAL;
+    if (device_buf && (!aligned16(device_buf) || is_host_ptr(device_buf)))
+        return fail(c, RC_E_INVAL, "the trace buffer must be 16-byte aligned device memory");
+    c->trace = static_cast<long long *>(device_buf);
+    c->trace_entries = device_buf ? bytes / sizeof(long long) : 0;
     return RC_OK;
 }
 

@@ -45,6 +45,7 @@ struct StepArgs {
     uint32_t n_steps;
     DevBlock *dev;
     cudaGraphConditionalHandle h_while;
+    long long *trace;        // optional per-step phase clocks of two CTAs (profiling), or null
 };
 
 // Epilogue flags of the per-step kernel.
@@ -76,6 +77,11 @@ cudaError_t launch_step(const StepArgs &a, int state_bytes, int payload_bytes, i
 // Persistent chains.  The single-CTA form takes K <= 1024; the grid form is a
 // cooperative launch of `grid` CTAs.
 cudaError_t launch_chain_cta(const StepArgs &a, int state_bytes, int payload_bytes, cudaStream_t s);
+// Pipelined single-CTA chains (identity sessions: records in registers;
+// explicit indices, 16-byte records, K <= 512: D-step prefetch with a shared
+// write-back table).  *launched is false when neither applies.
+cudaError_t launch_chain_cta_fast(const StepArgs &a, int state_bytes, int payload_bytes, cudaStream_t s,
+                                  bool *launched);
 cudaError_t chain_grid_size(int state_bytes, int payload_bytes, uint32_t K, int *grid);
 cudaError_t launch_chain_grid(const StepArgs &a, int state_bytes, int payload_bytes, int grid,
                               cudaStream_t s);

@@ -150,20 +150,48 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
     return done != 0u;
 }
 
-// 2-D tiled tensor load (box of the map) into shared memory, completing on bar.
-__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, int32_t x, int32_t y, uint64_t *bar) {
+// L2 eviction-priority policies (applied to whole accesses).
+__device__ __forceinline__ uint64_t policy_evict_first() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+__device__ __forceinline__ uint64_t policy_evict_last() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+
+__device__ __forceinline__ void tma_load_2d_hint(void *dst, const CUtensorMap *map, int32_t x, int32_t y,
+                                                 uint64_t *bar, uint64_t policy) {
     asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
-            smem_addr(dst)),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(smem_addr(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar)), "l"(policy)
         : "memory");
 }
 
-// Contiguous bulk copy global -> shared (16-byte aligned, size a multiple of 16).
-__device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
-    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                     smem_addr(dst)),
-                 "l"(src), "r"(bytes), "r"(smem_addr(bar))
+__device__ __forceinline__ void bulk_load_hint(void *dst, const void *src, uint32_t bytes, uint64_t *bar,
+                                               uint64_t policy) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::
+            "r"(smem_addr(dst)),
+        "l"(src), "r"(bytes), "r"(smem_addr(bar)), "l"(policy)
+        : "memory");
+}
+
+// 16-byte global load / store at L2 (L1 bypassed) with an L2 eviction policy.
+__device__ __forceinline__ uint4 ld_cg_hint(const uint4 *p, uint64_t policy) {
+    uint4 v;
+    asm volatile("ld.global.cg.L2::cache_hint.v4.u32 {%0, %1, %2, %3}, [%4], %5;"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p), "l"(policy)
+                 : "memory");
+    return v;
+}
+__device__ __forceinline__ void st_hint(uint4 *p, uint4 v, uint64_t policy) {
+    asm volatile("st.global.L2::cache_hint.v4.u32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(p), "r"(v.x), "r"(v.y),
+                 "r"(v.z), "r"(v.w), "l"(policy)
                  : "memory");
 }
 
@@ -176,6 +204,29 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 // Makes mbarrier initialisation visible to the async proxy.
 __device__ __forceinline__ void fence_mbar_init() {
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+// ---- per-thread asynchronous copies global -> shared (LDGSTS) ----------------
+__device__ __forceinline__ void cp_async4(void *dst, const void *src) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_addr(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async16(void *dst, const void *src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// Position of 16-byte chunk k of member m's payload in a per-member shared
+// ring: an XOR of the chunk index with bits of m so that the eight lanes of a
+// shared-memory phase hit eight different 16-byte bank groups.
+template <int P>
+__device__ __forceinline__ uint32_t pay_chunk(uint32_t m, uint32_t k) {
+    constexpr uint32_t nc = P / 16;                          // 2, 4 or 8 chunks
+    constexpr uint32_t shift = nc == 8 ? 0u : (nc == 4 ? 1u : 2u);
+    return m * nc + (k ^ ((m >> shift) & (nc - 1u)));
 }
 
 // Copies both route bodies' tables into shared memory (16-byte vectors).
@@ -209,9 +260,19 @@ __device__ __forceinline__ void load_event(Event<P> &ev, const StepArgs &a, uint
 // or a rejected member (error latched, nothing written).  `cg_state` reads the
 // state record at L2 (bypassing L1), as needed when other CTAs of a persistent
 // grid wrote it after this SM last cached it.
-template <int SB, int P, bool CG_STATE>
+// Deferred outputs of one member: the effect record and the new state record,
+// stored after the grid-barrier arrival (they are outputs only).
+template <int SB>
+struct Deferred {
+    uint4 eff;
+    uint4 rec[SB / 16];
+    bool valid;
+};
+
+template <int SB, int P, bool CG_STATE, bool HINT = false, bool DEFER = false>
 __device__ __forceinline__ uint32_t transition(const StepArgs &a, const Event<P> &ev, const uint8_t *tab,
-                                               uint32_t sel, uint32_t n, uint32_t m) {
+                                               uint32_t sel, uint32_t n, uint32_t m, uint64_t keep = 0,
+                                               Deferred<SB> *out = nullptr) {
     constexpr int NV = SB / 16;
     if (ev.s >= a.n_sessions) {
         latch_error(a.dev, DEV_E_INDEX, n, m);
@@ -220,7 +281,12 @@ __device__ __forceinline__ uint32_t transition(const StepArgs &a, const Event<P>
     uint4 *rp = reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(ev.s) * SB);
     uint4 r[NV];
 #pragma unroll
-    for (int k = 0; k < NV; ++k) r[k] = CG_STATE ? __ldcg(rp + k) : rp[k];
+    for (int k = 0; k < NV; ++k) {
+        if constexpr (HINT)
+            r[k] = ld_cg_hint(rp + k, keep);
+        else
+            r[k] = CG_STATE ? __ldcg(rp + k) : rp[k];
+    }
     const uint32_t x = r[0].x;
     if (x >= a.S || ev.o >= 8u) {
         latch_error(a.dev, DEV_E_STATE, n, m);
@@ -232,22 +298,44 @@ __device__ __forceinline__ uint32_t transition(const StepArgs &a, const Event<P>
     r[0].y = r[0].y + 1u;
     mix_acc<SB>(r, rk);
 #pragma unroll
-    for (int k = 0; k < NV; ++k) rp[k] = r[k];
-    const size_t slot = static_cast<size_t>(n) * a.K + m;
-    if (a.effects) {
-        uint4 e;
-        e.x = static_cast<uint32_t>(rk);
-        e.y = static_cast<uint32_t>(rk >> 32);
-        e.z = ev.s;
-        e.w = y | (ev.o << 16) | (sel << 24);
-        __stcs(reinterpret_cast<uint4 *>(a.effects) + slot, e);
+    for (int k = 0; k < NV; ++k) {
+        if constexpr (HINT)
+            st_hint(rp + k, r[k], keep);
+        else
+            rp[k] = r[k];
     }
+    uint4 e;
+    e.x = static_cast<uint32_t>(rk);
+    e.y = static_cast<uint32_t>(rk >> 32);
+    e.z = ev.s;
+    e.w = y | (ev.o << 16) | (sel << 24);
+    if constexpr (DEFER) {
+        out->eff = e;
+#pragma unroll
+        for (int k = 0; k < NV; ++k) out->rec[k] = r[k];
+        out->valid = true;
+    } else {
+        const size_t slot = static_cast<size_t>(n) * a.K + m;
+        if (a.effects) __stcs(reinterpret_cast<uint4 *>(a.effects) + slot, e);
+        if (a.state_log) {
+            uint4 *lp = reinterpret_cast<uint4 *>(a.state_log + slot * SB);
+#pragma unroll
+            for (int k = 0; k < NV; ++k) __stcs(lp + k, r[k]);
+        }
+    }
+    return static_cast<uint32_t>(rk & 1u);
+}
+
+template <int SB>
+__device__ __forceinline__ void store_deferred(const StepArgs &a, const Deferred<SB> &d, uint32_t n, uint32_t m) {
+    if (!d.valid) return;
+    const size_t slot = static_cast<size_t>(n) * a.K + m;
+    if (a.effects) __stcs(reinterpret_cast<uint4 *>(a.effects) + slot, d.eff);
     if (a.state_log) {
         uint4 *lp = reinterpret_cast<uint4 *>(a.state_log + slot * SB);
 #pragma unroll
-        for (int k = 0; k < NV; ++k) __stcs(lp + k, r[k]);
+        for (int k = 0; k < SB / 16; ++k) __stcs(lp + k, d.rec[k]);
     }
-    return static_cast<uint32_t>(rk & 1u);
 }
 
 // ---------------------------------------------------------------------------
@@ -337,6 +425,273 @@ __global__ void __launch_bounds__(1024) k_chain_cta(StepArgs a) {
     if (tid == 0) {
         if (a.n_steps > 0) a.dev->sel = sel;
         a.dev->step = a.n_steps;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Persistent chain, one CTA, 16-byte records, explicit session indices,
+// K <= 512: a D-step software pipeline.  At step n each thread copies (with
+// per-thread asynchronous copies into shared rings) the session index of its
+// member for step n + 2D, and the outcome, payload and session record for
+// step n + D.  The record fetched D steps early misses what steps n..n+D-1
+// write to that session; each step therefore keeps its new records and a
+// session -> member table in shared memory (one per step of the last D+1,
+// entries tagged with the step so no table is ever cleared), and step n takes
+// a session's record from the most recent of steps n-D..n-1 that wrote it,
+// else from its early copy.  The state array still receives every step's
+// records.  Per step the decision is reduced in shared memory and never
+// leaves the SM.
+// ---------------------------------------------------------------------------
+template <int P, int D>
+__global__ void __launch_bounds__(512, 1) k_chain_cta_pipe(StepArgs a, uint32_t tbl_bits) {
+    constexpr uint32_t RI = 2 * D + 1;  // index ring depth
+    constexpr uint32_t RD = D + 1;      // data, record and table ring depth
+    constexpr uint32_t NC = P / 16;
+    extern __shared__ __align__(16) uint8_t dsm[];
+    __shared__ uint32_t warp_odd[2][16];
+    const uint32_t K = a.K;
+    const uint32_t Kp = (K + 3u) & ~3u;
+    const uint32_t tid = threadIdx.x;
+    const uint32_t nw = (blockDim.x + 31u) / 32u;
+    const uint32_t slots = 1u << tbl_bits;
+    uint8_t *tab = dsm;
+    uint32_t *idx_r = reinterpret_cast<uint32_t *>(dsm + 2 * a.tab_stride);
+    uint32_t *out_r = idx_r + RI * Kp;
+    uint4 *pay_r = reinterpret_cast<uint4 *>(out_r + RD * Kp);
+    uint4 *gat_r = pay_r + RD * Kp * NC;
+    uint4 *rec_r = gat_r + RD * Kp;
+    unsigned long long *tbl = reinterpret_cast<unsigned long long *>(rec_r + RD * Kp);
+    uint16_t *tval = reinterpret_cast<uint16_t *>(tbl + RD * slots);
+
+    stage_tables(tab, a.tables, a.tab_stride, 2, 0);
+    for (uint32_t i = tid; i < RD * slots; i += blockDim.x) tbl[i] = ~0ull;
+    uint32_t sel = ld_volatile_u32(&a.dev->sel) & 1u;
+    const bool act = tid < K;
+    const uint32_t m = tid;
+    const uint32_t nst = a.n_steps;
+
+    auto ev_at = [&](uint32_t j) -> size_t { return static_cast<size_t>(j % a.n_sets) * K + m; };
+    auto issue_idx = [&](uint32_t j) {
+        if (act && j < nst) cp_async4(&idx_r[(j % RI) * Kp + m], a.idx + ev_at(j));
+    };
+    auto issue_data = [&](uint32_t j) {
+        if (!act || j >= nst) return;
+        const size_t e = ev_at(j);
+        cp_async4(&out_r[(j % RD) * Kp + m], a.outcome + e);
+        const uint4 *src = reinterpret_cast<const uint4 *>(a.payload + e * P);
+        uint4 *ring = pay_r + (j % RD) * Kp * NC;
+#pragma unroll
+        for (uint32_t k = 0; k < NC; ++k) cp_async16(ring + pay_chunk<P>(m, k), src + k);
+        const uint32_t sj = idx_r[(j % RI) * Kp + m];
+        if (sj < a.n_sessions) cp_async16(&gat_r[(j % RD) * Kp + m], a.state + static_cast<size_t>(sj) * 16);
+    };
+    auto hash = [&](uint32_t key) { return (key * 0x9E3779B1u) >> (32u - tbl_bits); };
+
+    for (uint32_t j = 0; j < 2u * D; ++j) issue_idx(j);
+    cp_async_commit();
+    cp_async_wait<0>();
+    for (uint32_t j = 0; j < D; ++j) {
+        issue_data(j);
+        cp_async_commit();
+    }
+    __syncthreads();
+
+    for (uint32_t n = 0; n < nst; ++n) {
+        cp_async_wait<D - 1>();  // this thread's copies for step n have landed
+        uint32_t odd = 0;
+        if (act) {
+            const uint32_t s = idx_r[(n % RI) * Kp + m];
+            const uint32_t o = out_r[(n % RD) * Kp + m];
+            if (s >= a.n_sessions) {
+                latch_error(a.dev, DEV_E_INDEX, n, m);
+            } else {
+                uint4 r = gat_r[(n % RD) * Kp + m];
+                // newest write among steps n-1 .. n-D wins over the early copy
+#pragma unroll
+                for (uint32_t dd = 1; dd <= D; ++dd) {
+                    if (n < dd) break;
+                    const uint32_t j = n - dd;
+                    const unsigned long long *tb = tbl + (j % RD) * slots;
+                    uint32_t h = hash(s);
+                    bool found = false;
+                    for (uint32_t probe = 0; probe < slots; ++probe) {
+                        const unsigned long long cur = tb[h];
+                        if (static_cast<uint32_t>(cur >> 32) != j) break;
+                        if (static_cast<uint32_t>(cur) == s) {
+                            r = rec_r[(j % RD) * Kp + tval[(j % RD) * slots + h]];
+                            found = true;
+                            break;
+                        }
+                        h = (h + 1u) & (slots - 1u);
+                    }
+                    if (found) break;
+                }
+                const uint32_t x = r.x;
+                if (x >= a.S || o >= 8u) {
+                    latch_error(a.dev, DEV_E_STATE, n, m);
+                } else {
+                    uint4 pw[NC];
+                    const uint4 *ring = pay_r + (n % RD) * Kp * NC;
+#pragma unroll
+                    for (uint32_t k = 0; k < NC; ++k) pw[k] = ring[pay_chunk<P>(m, k)];
+                    const uint64_t rk = route_key<P>(x, o, pw);
+                    const uint32_t y = tab[sel * a.tab_stride + x * 8u + o];
+                    uint4 rr[1] = {r};
+                    rr[0].x = y;
+                    rr[0].y = r.y + 1u;
+                    mix_acc<16>(rr, rk);
+                    r = rr[0];
+                    reinterpret_cast<uint4 *>(a.state)[s] = r;
+                    rec_r[(n % RD) * Kp + m] = r;
+                    unsigned long long *tb = tbl + (n % RD) * slots;
+                    const unsigned long long mine = (static_cast<unsigned long long>(n) << 32) | s;
+                    uint32_t h = hash(s);
+                    for (uint32_t probe = 0; probe < 2u * slots; ++probe) {
+                        const unsigned long long cur = tb[h];
+                        if (static_cast<uint32_t>(cur >> 32) != n) {
+                            if (atomicCAS(tb + h, cur, mine) == cur) {
+                                tval[(n % RD) * slots + h] = static_cast<uint16_t>(m);
+                                break;
+                            }
+                            continue;
+                        }
+                        h = (h + 1u) & (slots - 1u);
+                    }
+                    const size_t slot = static_cast<size_t>(n) * K + m;
+                    if (a.effects) {
+                        uint4 e;
+                        e.x = static_cast<uint32_t>(rk);
+                        e.y = static_cast<uint32_t>(rk >> 32);
+                        e.z = s;
+                        e.w = y | (o << 16) | (sel << 24);
+                        __stcs(reinterpret_cast<uint4 *>(a.effects) + slot, e);
+                    }
+                    if (a.state_log) __stcs(reinterpret_cast<uint4 *>(a.state_log) + slot, r);
+                    odd = static_cast<uint32_t>(rk & 1u);
+                }
+            }
+        }
+        issue_idx(n + 2u * D);
+        issue_data(n + D);
+        cp_async_commit();
+        const uint32_t ball = __ballot_sync(0xffffffffu, odd);
+        if ((tid & 31u) == 0) warp_odd[n & 1u][tid >> 5] = __popc(ball);
+        __syncthreads();  // also publishes this step's records and table to the next D steps
+        uint32_t total = 0;
+        for (uint32_t w = 0; w < nw; ++w) total += warp_odd[n & 1u][w];
+        sel = total > K / 2u ? 1u : 0u;
+        if (tid == 0 && a.decisions) a.decisions[n] = sel;
+    }
+    cp_async_wait<0>();
+    if (tid == 0) {
+        if (nst > 0) a.dev->sel = sel;
+        a.dev->step = nst;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Persistent chain, one CTA, member m is session m (no index array): each
+// thread keeps its session's record in registers for the whole chain and
+// writes it back once at the end (and to the state log per step when asked).
+// Outcomes and payloads stream through a D-deep ring of per-thread
+// asynchronous copies.
+// ---------------------------------------------------------------------------
+template <int SB, int P, int D>
+__global__ void __launch_bounds__(1024, 1) k_chain_cta_ident(StepArgs a) {
+    constexpr uint32_t RD = D + 1;
+    constexpr uint32_t NC = P / 16;
+    constexpr int NV = SB / 16;
+    extern __shared__ __align__(16) uint8_t dsm[];
+    __shared__ uint32_t warp_odd[2][32];
+    const uint32_t K = a.K;
+    const uint32_t Kp = (K + 3u) & ~3u;
+    const uint32_t tid = threadIdx.x;
+    const uint32_t nw = (blockDim.x + 31u) / 32u;
+    uint8_t *tab = dsm;
+    uint32_t *out_r = reinterpret_cast<uint32_t *>(dsm + 2 * a.tab_stride);
+    uint4 *pay_r = reinterpret_cast<uint4 *>(out_r + RD * Kp);
+    stage_tables(tab, a.tables, a.tab_stride, 2, 0);
+    uint32_t sel = ld_volatile_u32(&a.dev->sel) & 1u;
+    const bool act = tid < K;
+    const uint32_t m = tid;
+    const uint32_t nst = a.n_steps;
+    const bool in_range = m < a.n_sessions;
+    uint4 r[NV];
+    if (act && in_range) {
+        const uint4 *rp = reinterpret_cast<const uint4 *>(a.state + static_cast<size_t>(m) * SB);
+#pragma unroll
+        for (int k = 0; k < NV; ++k) r[k] = rp[k];
+    }
+    auto issue_data = [&](uint32_t j) {
+        if (!act || j >= nst) return;
+        const size_t e = static_cast<size_t>(j % a.n_sets) * K + m;
+        cp_async4(&out_r[(j % RD) * Kp + m], a.outcome + e);
+        const uint4 *src = reinterpret_cast<const uint4 *>(a.payload + e * P);
+        uint4 *ring = pay_r + (j % RD) * Kp * NC;
+#pragma unroll
+        for (uint32_t k = 0; k < NC; ++k) cp_async16(ring + pay_chunk<P>(m, k), src + k);
+    };
+    for (uint32_t j = 0; j < D; ++j) {
+        issue_data(j);
+        cp_async_commit();
+    }
+    __syncthreads();
+    for (uint32_t n = 0; n < nst; ++n) {
+        cp_async_wait<D - 1>();
+        uint32_t odd = 0;
+        if (act) {
+            const uint32_t o = out_r[(n % RD) * Kp + m];
+            if (!in_range) {
+                latch_error(a.dev, DEV_E_INDEX, n, m);
+            } else if (r[0].x >= a.S || o >= 8u) {
+                latch_error(a.dev, DEV_E_STATE, n, m);
+            } else {
+                uint4 pw[NC];
+                const uint4 *ring = pay_r + (n % RD) * Kp * NC;
+#pragma unroll
+                for (uint32_t k = 0; k < NC; ++k) pw[k] = ring[pay_chunk<P>(m, k)];
+                const uint32_t x = r[0].x;
+                const uint64_t rk = route_key<P>(x, o, pw);
+                const uint32_t y = tab[sel * a.tab_stride + x * 8u + o];
+                r[0].x = y;
+                r[0].y = r[0].y + 1u;
+                mix_acc<SB>(r, rk);
+                const size_t slot = static_cast<size_t>(n) * K + m;
+                if (a.effects) {
+                    uint4 e;
+                    e.x = static_cast<uint32_t>(rk);
+                    e.y = static_cast<uint32_t>(rk >> 32);
+                    e.z = m;
+                    e.w = y | (o << 16) | (sel << 24);
+                    __stcs(reinterpret_cast<uint4 *>(a.effects) + slot, e);
+                }
+                if (a.state_log) {
+                    uint4 *lp = reinterpret_cast<uint4 *>(a.state_log + slot * SB);
+#pragma unroll
+                    for (int k = 0; k < NV; ++k) __stcs(lp + k, r[k]);
+                }
+                odd = static_cast<uint32_t>(rk & 1u);
+            }
+        }
+        issue_data(n + D);
+        cp_async_commit();
+        const uint32_t ball = __ballot_sync(0xffffffffu, odd);
+        if ((tid & 31u) == 0) warp_odd[n & 1u][tid >> 5] = __popc(ball);
+        __syncthreads();
+        uint32_t total = 0;
+        for (uint32_t w = 0; w < nw; ++w) total += warp_odd[n & 1u][w];
+        sel = total > K / 2u ? 1u : 0u;
+        if (tid == 0 && a.decisions) a.decisions[n] = sel;
+    }
+    cp_async_wait<0>();
+    if (act && in_range) {
+        uint4 *rp = reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(m) * SB);
+#pragma unroll
+        for (int k = 0; k < NV; ++k) rp[k] = r[k];
+    }
+    if (tid == 0) {
+        if (nst > 0) a.dev->sel = sel;
+        a.dev->step = nst;
     }
 }
 
@@ -479,6 +834,15 @@ __global__ void __launch_bounds__(512, 1)
     const uint32_t m0 = blockIdx.x * sh.chunk;
     const uint32_t cnt = m0 < a.K ? min(sh.chunk, a.K - m0) : 0u;
     const uint64_t limit = a.dev->wait_ns;
+    // event streams are read once: evict them first; session records are
+    // re-read by later steps: keep them
+    const uint64_t stream_pol = policy_evict_first();
+    const uint64_t keep_pol = policy_evict_last();
+    const uint32_t issuer = blockDim.x > 32u ? 32u : 0u;  // lane 0 of warp 1 issues the copies
+    // profiling: thread 0 of the first and last CTA records six phase clocks per step
+    long long *trace = (a.trace && tid == 0 && (blockIdx.x == 0 || blockIdx.x == gridDim.x - 1))
+                           ? a.trace + (blockIdx.x == 0 ? 0 : static_cast<size_t>(a.n_steps) * 6)
+                           : nullptr;
 
     // thread 0 issues the copies of step j into stage j & 1
     auto issue = [&](uint32_t j) {
@@ -487,10 +851,10 @@ __global__ void __launch_bounds__(512, 1)
         const uint32_t bytes = sh.n_boxes * sh.box_rows * P + cnt * 4u * (a.idx ? 2u : 1u);
         mbar_arrive_expect_tx(&bar[st], bytes);
         for (uint32_t b = 0; b < sh.n_boxes; ++b)
-            tma_load_2d(pay_of(st) + b * sh.box_rows * P, &tmap, 0, static_cast<int32_t>(row0 + b * sh.box_rows),
-                        &bar[st]);
-        bulk_load(out_of(st), a.outcome + row0, cnt * 4u, &bar[st]);
-        if (a.idx) bulk_load(idx_of(st), a.idx + row0, cnt * 4u, &bar[st]);
+            tma_load_2d_hint(pay_of(st) + b * sh.box_rows * P, &tmap, 0,
+                             static_cast<int32_t>(row0 + b * sh.box_rows), &bar[st], stream_pol);
+        bulk_load_hint(out_of(st), a.outcome + row0, cnt * 4u, &bar[st], stream_pol);
+        if (a.idx) bulk_load_hint(idx_of(st), a.idx + row0, cnt * 4u, &bar[st], stream_pol);
         s_pending |= 1u << st;
         s_pend_step[st] = j;
     };
@@ -522,6 +886,7 @@ __global__ void __launch_bounds__(512, 1)
     for (uint32_t n = 0; n < a.n_steps; ++n) {
         const uint32_t st = n & 1u;
         uint32_t odd = 0;
+        if (trace) trace[n * 6 + 0] = clock64();
         if (cnt > 0) {
             if (!wait_stage(st, (n >> 1) & 1u)) {
                 latch_error(a.dev, DEV_E_TIMEOUT, n, blockIdx.x);
@@ -531,12 +896,20 @@ __global__ void __launch_bounds__(512, 1)
         }
         __syncthreads();
         if (s_abort) break;
+        if (trace) trace[n * 6 + 1] = clock64();
+        const bool one_each = cnt <= blockDim.x;  // one member per thread: outputs can wait
+        Deferred<SB> dfr;
+        dfr.valid = false;
         for (uint32_t t = tid; t < cnt; t += blockDim.x) {
             Event<P> ev;
             ev.s = a.idx ? idx_of(st)[t] : m0 + t;
             ev.o = out_of(st)[t];
             read_payload_swizzled<P>(ev.pw, pay_of(st), t);
-            odd += transition<SB, P, true>(a, ev, tab + sel * a.tab_stride, sel, n, m0 + t);
+            if (one_each)
+                odd += transition<SB, P, true, true, true>(a, ev, tab + sel * a.tab_stride, sel, n, m0 + t,
+                                                           keep_pol, &dfr);
+            else
+                odd += transition<SB, P, true, true>(a, ev, tab + sel * a.tab_stride, sel, n, m0 + t, keep_pol);
         }
         uint32_t v = odd;
 #pragma unroll
@@ -544,7 +917,7 @@ __global__ void __launch_bounds__(512, 1)
         if ((tid & 31u) == 0) warp_odd[tid >> 5] = v;
         __syncthreads();  // every thread is done with stage st and has stored this step's records
         if (tid == 0) {
-            if (cnt > 0) s_pending &= ~(1u << st);
+            if (trace) trace[n * 6 + 2] = clock64();
             uint32_t c = 0;
             for (uint32_t w = 0; w < (blockDim.x + 31u) / 32u; ++w) c += warp_odd[w];
             unsigned long long *word = &a.dev->slot[n % 3u];
@@ -552,10 +925,15 @@ __global__ void __launch_bounds__(512, 1)
             __threadfence();
             const bool skip = (n == 0 && blockIdx.x == 1 && ld_volatile_u32(&a.dev->skip_arrival) != 0u);
             if (!skip) red_release_add_u64(word, (1ull << 32) | c);
-            if (cnt > 0 && n + 2u < a.n_steps) {
-                fence_proxy_async_smem();
-                issue(n + 2u);
+            if (trace) trace[n * 6 + 3] = clock64();
+            if (issuer == 0) {
+                if (cnt > 0) s_pending &= ~(1u << st);
+                if (cnt > 0 && n + 2u < a.n_steps) {
+                    fence_proxy_async_smem();
+                    issue(n + 2u);
+                }
             }
+            if (trace) trace[n * 6 + 4] = clock64();
             const uint64_t t0 = globaltimer_ns();
             unsigned long long w;
             uint32_t spins = 0;
@@ -576,10 +954,19 @@ __global__ void __launch_bounds__(512, 1)
                 }
             }
             __threadfence();
+            if (trace) trace[n * 6 + 5] = clock64();
             const uint32_t d = (static_cast<uint32_t>(w & 0xffffffffull) > a.K / 2u) ? 1u : 0u;
             s_sel = d;
             if (blockIdx.x == 0 && a.decisions && !s_abort) a.decisions[n] = d;
+        } else if (tid == issuer) {
+            // the copies for step n + 2 go out while thread 0 arrives and waits
+            if (cnt > 0) s_pending &= ~(1u << st);
+            if (cnt > 0 && n + 2u < a.n_steps) {
+                fence_proxy_async_smem();
+                issue(n + 2u);
+            }
         }
+        if (one_each) store_deferred<SB>(a, dfr, n, m0 + tid);
         __syncthreads();
         if (s_abort) break;
         sel = s_sel;
@@ -676,6 +1063,77 @@ cudaError_t launch_step(const StepArgs &a, int SB, int P, int step, int sel, uin
     StepArgs aa = a;
     void *args[] = {&aa, &step, &sel, &epi};
     return cudaLaunchKernel(fn, step_grid(a.K), step_block(a.K), args, 0, s);
+}
+
+namespace {
+template <int P, int D>
+const void *pipe_fn() {
+    return reinterpret_cast<const void *>(&k_chain_cta_pipe<P, D>);
+}
+template <int SB, int P, int D>
+const void *ident_fn() {
+    return reinterpret_cast<const void *>(&k_chain_cta_ident<SB, P, D>);
+}
+const void *pipe_fn_rt(int P, int D) {
+    if (D == 4) return P == 32 ? pipe_fn<32, 4>() : P == 64 ? pipe_fn<64, 4>() : pipe_fn<128, 4>();
+    return P == 32 ? pipe_fn<32, 2>() : P == 64 ? pipe_fn<64, 2>() : pipe_fn<128, 2>();
+}
+const void *ident_fn_rt(int SB, int P, int D) {
+    return dispatch(SB, P, [&](auto b, auto q) {
+        constexpr int B = decltype(b)::value, Q = decltype(q)::value;
+        return D == 4 ? ident_fn<B, Q, 4>() : D == 2 ? ident_fn<B, Q, 2>() : ident_fn<B, Q, 1>();
+    });
+}
+size_t pipe_smem(uint32_t K, int P, int D, uint32_t tab_stride, uint32_t tbl_bits) {
+    const size_t Kp = (K + 3u) & ~3u, RI = 2 * D + 1, RD = D + 1, slots = size_t(1) << tbl_bits;
+    return 2 * tab_stride + RI * Kp * 4 + RD * Kp * 4 + RD * Kp * P + 2 * RD * Kp * 16 + RD * slots * 10;
+}
+size_t ident_smem(uint32_t K, int P, int D, uint32_t tab_stride) {
+    const size_t Kp = (K + 3u) & ~3u, RD = D + 1;
+    return 2 * tab_stride + RD * Kp * 4 + RD * Kp * P;
+}
+int max_optin_smem() {
+    int dev = 0, v = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess) return 0;
+    return v;
+}
+}  // namespace
+
+cudaError_t launch_chain_cta_fast(const StepArgs &a, int SB, int P, cudaStream_t s, bool *launched) {
+    *launched = false;
+    const uint32_t K = a.K;
+    if (K == 0 || K > 1024u) return cudaSuccess;
+    const size_t cap = static_cast<size_t>(max_optin_smem());
+    const uint32_t threads = ((K + 31u) / 32u) * 32u;
+    StepArgs aa = a;
+    if (!a.idx) {
+        for (int D : {4, 2, 1}) {
+            const size_t smem = ident_smem(K, P, D, a.tab_stride);
+            if (smem > cap) continue;
+            const void *fn = ident_fn_rt(SB, P, D);
+            cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+            if (e != cudaSuccess) return e;
+            void *args[] = {&aa};
+            *launched = true;
+            return cudaLaunchKernel(fn, dim3(1), dim3(threads), args, smem, s);
+        }
+        return cudaSuccess;
+    }
+    if (SB != 16 || K > 512u) return cudaSuccess;
+    uint32_t tbl_bits = 1;
+    while ((1u << tbl_bits) < 2u * K) ++tbl_bits;
+    for (int D : {4, 2}) {
+        const size_t smem = pipe_smem(K, P, D, a.tab_stride, tbl_bits);
+        if (smem > cap) continue;
+        const void *fn = pipe_fn_rt(P, D);
+        cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+        if (e != cudaSuccess) return e;
+        void *args[] = {&aa, &tbl_bits};
+        *launched = true;
+        return cudaLaunchKernel(fn, dim3(1), dim3(threads), args, smem, s);
+    }
+    return cudaSuccess;
 }
 
 cudaError_t launch_chain_cta(const StepArgs &a, int SB, int P, cudaStream_t s) {

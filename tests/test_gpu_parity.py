@@ -213,3 +213,30 @@ def test_grid_barrier_wait_is_bounded_both_kernels(g, rc, monkeypatch, tma):
         assert np.array_equal(g.host(state, np.uint8).reshape(state0.shape), want["state"])
     finally:
         rc.rc_free(ctx)
+
+
+@pytest.mark.parametrize("pipe", [True, False])
+@pytest.mark.parametrize("P", [32, 64, 128])
+@pytest.mark.parametrize("K,N", [(8, 9), (64, 67), (64, 128), (256, 259), (256, 512), (500, 1000), (512, 513)])
+def test_single_cta_pipeline_repeated_sessions(g, rc, monkeypatch, pipe, P, K, N):
+    """Sessions that recur in consecutive steps at other member positions: the
+    pipelined kernel must take their records from the steps that just wrote
+    them, not from its early copies."""
+    monkeypatch.setenv("RC_NO_PIPE", "0" if pipe else "1")
+    tables, state0, outc, pay, idx = _inputs(60 + K % 13 + P, K, 64, 16, P, 40, N=N)
+    n = 40
+    want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=1)
+    got = g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K, sel0=1)
+    g.assert_same(got, want, f"pipe={pipe} K={K} N={N} P={P}")
+
+
+@pytest.mark.parametrize("pipe", [True, False])
+@pytest.mark.parametrize("SB,P,K", [(16, 32, 32), (16, 32, 256), (64, 128, 256), (64, 64, 700), (16, 128, 1024)])
+def test_single_cta_identity_sessions(g, rc, monkeypatch, pipe, SB, P, K):
+    monkeypatch.setenv("RC_NO_PIPE", "0" if pipe else "1")
+    S = 256 if SB == 64 else 128
+    tables, state0, outc, pay, idx = _inputs(80 + K % 17, K, S, SB, P, 30)
+    n = 30
+    want = g.run_oracle(tables, state0, outc, pay, idx, n)
+    got = g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K)
+    g.assert_same(got, want, f"identity pipe={pipe} SB={SB} P={P} K={K}")
