@@ -88,7 +88,9 @@ struct rc_ctx {
     double last_ms = 0.0;
     uint32_t last_launches = 0;
     bool no_tma = false;   // RC_NO_TMA=1 in the environment selects the plain grid kernel
-    bool no_pipe = false;  // RC_NO_PIPE=1 selects the plain single-CTA kernel
+    bool no_pipe = false;   // RC_NO_PIPE=1 selects the plain single-CTA kernel
+    bool no_split = false;  // RC_NO_SPLIT=1 turns the split-phase chain off
+    Buf marks;              // split-phase cohort marks (3 * n_sessions words)
     long long *trace = nullptr;
     uint64_t trace_entries = 0;
 };
@@ -373,6 +375,24 @@ int run_cond(rc_ctx *c, const rc::StepArgs &a) {
 
 // ---- device resident: persistent kernel ------------------------------------
 int run_persist(rc_ctx *c, const rc::StepArgs &a) {
+    if (a.idx && !c->no_split) {
+        int grid = 0;
+        uint32_t threads = 0;
+        size_t smem = 0;
+        alignas(8) unsigned char shape[32];
+        if (rc::chain_split_plan(c->SB, c->P, a.K, c->tab_stride, &grid, &threads, &smem, shape)) {
+            if (grid > 1 && !c->coop) return fail(c, RC_E_UNSUPPORTED, "device lacks cooperative launch");
+            int rc = ensure(c, c->marks, 3ull * c->n_sessions * sizeof(uint32_t));
+            if (rc != RC_OK) return rc;
+            RC_CUDA(c, cudaMemsetAsync(c->marks.p, 0xff, 3ull * c->n_sessions * sizeof(uint32_t), c->stream));
+            RC_CUDA(c, cudaMemsetAsync(c->dev->slot, 0, sizeof(c->dev->slot), c->stream));
+            RC_CUDA(c, cudaMemsetAsync(&c->dev->abort, 0, sizeof(uint32_t), c->stream));
+            RC_CUDA(c, rc::launch_chain_split(a, c->SB, c->P, grid, threads, smem, shape,
+                                              static_cast<uint32_t *>(c->marks.p), c->stream));
+            RC_CUDA(c, cudaMemsetAsync(&c->dev->skip_arrival, 0, sizeof(uint32_t), c->stream));
+            return RC_OK;
+        }
+    }
     if (a.K <= 1024u) {
         bool launched = false;
         if (!c->no_pipe) RC_CUDA(c, rc::launch_chain_cta_fast(a, c->SB, c->P, c->stream, &launched));
@@ -511,6 +531,8 @@ int rc_init(rc_ctx **out, uint32_t S, const uint8_t *table, uint32_t state_bytes
         c->no_tma = v && v[0] == '1';
         const char *w = std::getenv("RC_NO_PIPE");
         c->no_pipe = w && w[0] == '1';
+        const char *x = std::getenv("RC_NO_SPLIT");
+        c->no_split = x && x[0] == '1';
     }
     auto bail = [&](cudaError_t e) {
         rc_free(c);
@@ -614,7 +636,7 @@ int rc_free(rc_ctx *c) {
     c->cond.reset();
     c->floor.reset();
     c->nested.reset();
-    for (Buf *b : {&c->st_outcome, &c->st_payload, &c->st_idx, &c->st_dec, &c->st_eff, &c->st_log})
+    for (Buf *b : {&c->st_outcome, &c->st_payload, &c->st_idx, &c->st_dec, &c->st_eff, &c->st_log, &c->marks})
         if (b->p) cudaFree(b->p);
     if (c->d_tables) cudaFree(c->d_tables);
     if (c->dev) cudaFree(c->dev);

@@ -93,6 +93,14 @@ bool chain_grid_tma_plan(int state_bytes, int payload_bytes, uint32_t K, uint32_
 cudaError_t launch_chain_grid_tma(const StepArgs &a, int state_bytes, int payload_bytes, int grid, uint32_t threads,
                                   size_t smem, const void *shape, cudaStream_t s);
 
+// Split-phase persistent chain (explicit session indices, K a multiple of 8,
+// at most 512 members per CTA): marks is device scratch of 3 * n_sessions
+// words, filled with 0xFF bytes before each launch.
+bool chain_split_plan(int state_bytes, int payload_bytes, uint32_t K, uint32_t tab_stride, int *grid,
+                      uint32_t *threads, size_t *smem, void *shape_out);
+cudaError_t launch_chain_split(const StepArgs &a, int state_bytes, int payload_bytes, int grid, uint32_t threads,
+                               size_t smem, const void *shape, uint32_t *marks, cudaStream_t s);
+
 // Writes decisions[0..n) = 0 and sel = 0 (an empty cohort decides 0).
 cudaError_t launch_empty_cohorts(const StepArgs &a, cudaStream_t s);
 

@@ -260,19 +260,9 @@ __device__ __forceinline__ void load_event(Event<P> &ev, const StepArgs &a, uint
 // or a rejected member (error latched, nothing written).  `cg_state` reads the
 // state record at L2 (bypassing L1), as needed when other CTAs of a persistent
 // grid wrote it after this SM last cached it.
-// Deferred outputs of one member: the effect record and the new state record,
-// stored after the grid-barrier arrival (they are outputs only).
-template <int SB>
-struct Deferred {
-    uint4 eff;
-    uint4 rec[SB / 16];
-    bool valid;
-};
-
-template <int SB, int P, bool CG_STATE, bool HINT = false, bool DEFER = false>
+template <int SB, int P, bool CG_STATE, bool HINT = false>
 __device__ __forceinline__ uint32_t transition(const StepArgs &a, const Event<P> &ev, const uint8_t *tab,
-                                               uint32_t sel, uint32_t n, uint32_t m, uint64_t keep = 0,
-                                               Deferred<SB> *out = nullptr) {
+                                               uint32_t sel, uint32_t n, uint32_t m, uint64_t keep = 0) {
     constexpr int NV = SB / 16;
     if (ev.s >= a.n_sessions) {
         latch_error(a.dev, DEV_E_INDEX, n, m);
@@ -304,38 +294,21 @@ __device__ __forceinline__ uint32_t transition(const StepArgs &a, const Event<P>
         else
             rp[k] = r[k];
     }
-    uint4 e;
-    e.x = static_cast<uint32_t>(rk);
-    e.y = static_cast<uint32_t>(rk >> 32);
-    e.z = ev.s;
-    e.w = y | (ev.o << 16) | (sel << 24);
-    if constexpr (DEFER) {
-        out->eff = e;
-#pragma unroll
-        for (int k = 0; k < NV; ++k) out->rec[k] = r[k];
-        out->valid = true;
-    } else {
-        const size_t slot = static_cast<size_t>(n) * a.K + m;
-        if (a.effects) __stcs(reinterpret_cast<uint4 *>(a.effects) + slot, e);
-        if (a.state_log) {
-            uint4 *lp = reinterpret_cast<uint4 *>(a.state_log + slot * SB);
-#pragma unroll
-            for (int k = 0; k < NV; ++k) __stcs(lp + k, r[k]);
-        }
-    }
-    return static_cast<uint32_t>(rk & 1u);
-}
-
-template <int SB>
-__device__ __forceinline__ void store_deferred(const StepArgs &a, const Deferred<SB> &d, uint32_t n, uint32_t m) {
-    if (!d.valid) return;
     const size_t slot = static_cast<size_t>(n) * a.K + m;
-    if (a.effects) __stcs(reinterpret_cast<uint4 *>(a.effects) + slot, d.eff);
+    if (a.effects) {
+        uint4 e;
+        e.x = static_cast<uint32_t>(rk);
+        e.y = static_cast<uint32_t>(rk >> 32);
+        e.z = ev.s;
+        e.w = y | (ev.o << 16) | (sel << 24);
+        __stcs(reinterpret_cast<uint4 *>(a.effects) + slot, e);
+    }
     if (a.state_log) {
         uint4 *lp = reinterpret_cast<uint4 *>(a.state_log + slot * SB);
 #pragma unroll
-        for (int k = 0; k < SB / 16; ++k) __stcs(lp + k, d.rec[k]);
+        for (int k = 0; k < NV; ++k) __stcs(lp + k, r[k]);
     }
+    return static_cast<uint32_t>(rk & 1u);
 }
 
 // ---------------------------------------------------------------------------
@@ -425,167 +398,6 @@ __global__ void __launch_bounds__(1024) k_chain_cta(StepArgs a) {
     if (tid == 0) {
         if (a.n_steps > 0) a.dev->sel = sel;
         a.dev->step = a.n_steps;
-    }
-}
-
-// ---------------------------------------------------------------------------
-// Persistent chain, one CTA, 16-byte records, explicit session indices,
-// K <= 512: a D-step software pipeline.  At step n each thread copies (with
-// per-thread asynchronous copies into shared rings) the session index of its
-// member for step n + 2D, and the outcome, payload and session record for
-// step n + D.  The record fetched D steps early misses what steps n..n+D-1
-// write to that session; each step therefore keeps its new records and a
-// session -> member table in shared memory (one per step of the last D+1,
-// entries tagged with the step so no table is ever cleared), and step n takes
-// a session's record from the most recent of steps n-D..n-1 that wrote it,
-// else from its early copy.  The state array still receives every step's
-// records.  Per step the decision is reduced in shared memory and never
-// leaves the SM.
-// ---------------------------------------------------------------------------
-template <int P, int D>
-__global__ void __launch_bounds__(512, 1) k_chain_cta_pipe(StepArgs a, uint32_t tbl_bits) {
-    constexpr uint32_t RI = 2 * D + 1;  // index ring depth
-    constexpr uint32_t RD = D + 1;      // data, record and table ring depth
-    constexpr uint32_t NC = P / 16;
-    extern __shared__ __align__(16) uint8_t dsm[];
-    __shared__ uint32_t warp_odd[2][16];
-    const uint32_t K = a.K;
-    const uint32_t Kp = (K + 3u) & ~3u;
-    const uint32_t tid = threadIdx.x;
-    const uint32_t nw = (blockDim.x + 31u) / 32u;
-    const uint32_t slots = 1u << tbl_bits;
-    uint8_t *tab = dsm;
-    uint32_t *idx_r = reinterpret_cast<uint32_t *>(dsm + 2 * a.tab_stride);
-    uint32_t *out_r = idx_r + RI * Kp;
-    uint4 *pay_r = reinterpret_cast<uint4 *>(out_r + RD * Kp);
-    uint4 *gat_r = pay_r + RD * Kp * NC;
-    uint4 *rec_r = gat_r + RD * Kp;
-    unsigned long long *tbl = reinterpret_cast<unsigned long long *>(rec_r + RD * Kp);
-    uint16_t *tval = reinterpret_cast<uint16_t *>(tbl + RD * slots);
-
-    stage_tables(tab, a.tables, a.tab_stride, 2, 0);
-    for (uint32_t i = tid; i < RD * slots; i += blockDim.x) tbl[i] = ~0ull;
-    uint32_t sel = ld_volatile_u32(&a.dev->sel) & 1u;
-    const bool act = tid < K;
-    const uint32_t m = tid;
-    const uint32_t nst = a.n_steps;
-
-    auto ev_at = [&](uint32_t j) -> size_t { return static_cast<size_t>(j % a.n_sets) * K + m; };
-    auto issue_idx = [&](uint32_t j) {
-        if (act && j < nst) cp_async4(&idx_r[(j % RI) * Kp + m], a.idx + ev_at(j));
-    };
-    auto issue_data = [&](uint32_t j) {
-        if (!act || j >= nst) return;
-        const size_t e = ev_at(j);
-        cp_async4(&out_r[(j % RD) * Kp + m], a.outcome + e);
-        const uint4 *src = reinterpret_cast<const uint4 *>(a.payload + e * P);
-        uint4 *ring = pay_r + (j % RD) * Kp * NC;
-#pragma unroll
-        for (uint32_t k = 0; k < NC; ++k) cp_async16(ring + pay_chunk<P>(m, k), src + k);
-        const uint32_t sj = idx_r[(j % RI) * Kp + m];
-        if (sj < a.n_sessions) cp_async16(&gat_r[(j % RD) * Kp + m], a.state + static_cast<size_t>(sj) * 16);
-    };
-    auto hash = [&](uint32_t key) { return (key * 0x9E3779B1u) >> (32u - tbl_bits); };
-
-    for (uint32_t j = 0; j < 2u * D; ++j) issue_idx(j);
-    cp_async_commit();
-    cp_async_wait<0>();
-    for (uint32_t j = 0; j < D; ++j) {
-        issue_data(j);
-        cp_async_commit();
-    }
-    __syncthreads();
-
-    for (uint32_t n = 0; n < nst; ++n) {
-        cp_async_wait<D - 1>();  // this thread's copies for step n have landed
-        uint32_t odd = 0;
-        if (act) {
-            const uint32_t s = idx_r[(n % RI) * Kp + m];
-            const uint32_t o = out_r[(n % RD) * Kp + m];
-            if (s >= a.n_sessions) {
-                latch_error(a.dev, DEV_E_INDEX, n, m);
-            } else {
-                uint4 r = gat_r[(n % RD) * Kp + m];
-                // newest write among steps n-1 .. n-D wins over the early copy
-#pragma unroll
-                for (uint32_t dd = 1; dd <= D; ++dd) {
-                    if (n < dd) break;
-                    const uint32_t j = n - dd;
-                    const unsigned long long *tb = tbl + (j % RD) * slots;
-                    uint32_t h = hash(s);
-                    bool found = false;
-                    for (uint32_t probe = 0; probe < slots; ++probe) {
-                        const unsigned long long cur = tb[h];
-                        if (static_cast<uint32_t>(cur >> 32) != j) break;
-                        if (static_cast<uint32_t>(cur) == s) {
-                            r = rec_r[(j % RD) * Kp + tval[(j % RD) * slots + h]];
-                            found = true;
-                            break;
-                        }
-                        h = (h + 1u) & (slots - 1u);
-                    }
-                    if (found) break;
-                }
-                const uint32_t x = r.x;
-                if (x >= a.S || o >= 8u) {
-                    latch_error(a.dev, DEV_E_STATE, n, m);
-                } else {
-                    uint4 pw[NC];
-                    const uint4 *ring = pay_r + (n % RD) * Kp * NC;
-#pragma unroll
-                    for (uint32_t k = 0; k < NC; ++k) pw[k] = ring[pay_chunk<P>(m, k)];
-                    const uint64_t rk = route_key<P>(x, o, pw);
-                    const uint32_t y = tab[sel * a.tab_stride + x * 8u + o];
-                    uint4 rr[1] = {r};
-                    rr[0].x = y;
-                    rr[0].y = r.y + 1u;
-                    mix_acc<16>(rr, rk);
-                    r = rr[0];
-                    reinterpret_cast<uint4 *>(a.state)[s] = r;
-                    rec_r[(n % RD) * Kp + m] = r;
-                    unsigned long long *tb = tbl + (n % RD) * slots;
-                    const unsigned long long mine = (static_cast<unsigned long long>(n) << 32) | s;
-                    uint32_t h = hash(s);
-                    for (uint32_t probe = 0; probe < 2u * slots; ++probe) {
-                        const unsigned long long cur = tb[h];
-                        if (static_cast<uint32_t>(cur >> 32) != n) {
-                            if (atomicCAS(tb + h, cur, mine) == cur) {
-                                tval[(n % RD) * slots + h] = static_cast<uint16_t>(m);
-                                break;
-                            }
-                            continue;
-                        }
-                        h = (h + 1u) & (slots - 1u);
-                    }
-                    const size_t slot = static_cast<size_t>(n) * K + m;
-                    if (a.effects) {
-                        uint4 e;
-                        e.x = static_cast<uint32_t>(rk);
-                        e.y = static_cast<uint32_t>(rk >> 32);
-                        e.z = s;
-                        e.w = y | (o << 16) | (sel << 24);
-                        __stcs(reinterpret_cast<uint4 *>(a.effects) + slot, e);
-                    }
-                    if (a.state_log) __stcs(reinterpret_cast<uint4 *>(a.state_log) + slot, r);
-                    odd = static_cast<uint32_t>(rk & 1u);
-                }
-            }
-        }
-        issue_idx(n + 2u * D);
-        issue_data(n + D);
-        cp_async_commit();
-        const uint32_t ball = __ballot_sync(0xffffffffu, odd);
-        if ((tid & 31u) == 0) warp_odd[n & 1u][tid >> 5] = __popc(ball);
-        __syncthreads();  // also publishes this step's records and table to the next D steps
-        uint32_t total = 0;
-        for (uint32_t w = 0; w < nw; ++w) total += warp_odd[n & 1u][w];
-        sel = total > K / 2u ? 1u : 0u;
-        if (tid == 0 && a.decisions) a.decisions[n] = sel;
-    }
-    cp_async_wait<0>();
-    if (tid == 0) {
-        if (nst > 0) a.dev->sel = sel;
-        a.dev->step = nst;
     }
 }
 
@@ -897,19 +709,12 @@ __global__ void __launch_bounds__(512, 1)
         __syncthreads();
         if (s_abort) break;
         if (trace) trace[n * 6 + 1] = clock64();
-        const bool one_each = cnt <= blockDim.x;  // one member per thread: outputs can wait
-        Deferred<SB> dfr;
-        dfr.valid = false;
         for (uint32_t t = tid; t < cnt; t += blockDim.x) {
             Event<P> ev;
             ev.s = a.idx ? idx_of(st)[t] : m0 + t;
             ev.o = out_of(st)[t];
             read_payload_swizzled<P>(ev.pw, pay_of(st), t);
-            if (one_each)
-                odd += transition<SB, P, true, true, true>(a, ev, tab + sel * a.tab_stride, sel, n, m0 + t,
-                                                           keep_pol, &dfr);
-            else
-                odd += transition<SB, P, true, true>(a, ev, tab + sel * a.tab_stride, sel, n, m0 + t, keep_pol);
+            odd += transition<SB, P, true, true>(a, ev, tab + sel * a.tab_stride, sel, n, m0 + t, keep_pol);
         }
         uint32_t v = odd;
 #pragma unroll
@@ -966,7 +771,6 @@ __global__ void __launch_bounds__(512, 1)
                 issue(n + 2u);
             }
         }
-        if (one_each) store_deferred<SB>(a, dfr, n, m0 + tid);
         __syncthreads();
         if (s_abort) break;
         sel = s_sel;
@@ -989,6 +793,269 @@ __global__ void __launch_bounds__(512, 1)
     }
     if (blockIdx.x == 0 && tid == 0) {
         if (a.n_steps > 0) a.dev->sel = sel;
+        a.dev->step = a.n_steps;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Persistent chain, split-phase (explicit session indices, K a multiple of 8,
+// at most 512 members per CTA; one CTA when K <= 512, else one CTA per SM).
+//
+// A member whose session is not in the previous cohort ("clean") does not
+// depend on that cohort's writes: its record, route key, odd bit, step and
+// accumulator can be computed one step early, while the previous step's
+// barrier resolves; only its next state y = T_sel[x][o] must wait for the
+// decision.  A member whose session is in the previous cohort ("dirty") is
+// gathered and hashed after that step's barrier.  Membership is found with
+// step-tagged marks in device scratch (three arrays, one per step mod 3; a
+// cohort's marks are written before the barrier that precedes any check
+// against them, and a CTA can run at most one barrier ahead, so a check never
+// meets a rewrite).  Iteration n (n = -1 .. n_steps - 1):
+//   A  finish the clean members of step n (table lookup, stores, effect);
+//      write the marks of cohort n + 1;
+//   B  gather, hash and finish the dirty members of step n (compacted list);
+//   -- CTA sync; thread 0 arrives at the grid barrier with the odd count of
+//      step n (the early count of its clean members + the dirty ones);
+//   C  early work for the clean members of step n + 1 (mark check, gather,
+//      route key, accumulator), overlapping the barrier wait;
+//   -- CTA sync after the barrier: the decision of step n selects the body
+//      of step n + 1.
+// Events arrive by TMA as in k_chain_grid_tma.  All waits are bounded.
+// ---------------------------------------------------------------------------
+template <int SB, int P>
+__global__ void __launch_bounds__(512, 1)
+    k_chain_split(const __grid_constant__ CUtensorMap tmap, StepArgs a, TmaShape sh, uint32_t *marks) {
+    constexpr int NV = SB / 16;
+    extern __shared__ uint8_t dsm_raw[];
+    __shared__ __align__(8) uint64_t bar[2];
+    __shared__ uint32_t warp_odd[16];
+    __shared__ uint16_t dlist[2][512];
+    __shared__ uint32_t dcount[2];
+    __shared__ uint32_t s_sel, s_abort, s_pending, s_pend_step[2];
+    const uint32_t raw = smem_addr(dsm_raw);
+    uint8_t *const base = dsm_raw + (((raw + 1023u) & ~1023u) - raw);
+    uint32_t *const words = reinterpret_cast<uint32_t *>(base + 2 * sh.stage_pay);
+    uint8_t *const tab = reinterpret_cast<uint8_t *>(words + 4 * sh.stage_words);
+    auto pay_of = [&](uint32_t st) { return base + st * sh.stage_pay; };
+    auto out_of = [&](uint32_t st) { return words + st * sh.stage_words; };
+    auto idx_of = [&](uint32_t st) { return words + (2u + st) * sh.stage_words; };
+
+    const uint32_t tid = threadIdx.x;
+    const uint32_t m0 = blockIdx.x * sh.chunk;
+    const uint32_t cnt = m0 < a.K ? min(sh.chunk, a.K - m0) : 0u;
+    const bool mine = tid < cnt;
+    const bool single = gridDim.x == 1;
+    const uint64_t limit = a.dev->wait_ns;
+    const uint64_t stream_pol = policy_evict_first();
+    const uint64_t keep_pol = policy_evict_last();
+    const uint32_t issuer = blockDim.x > 32u ? 32u : 0u;
+    const uint64_t N = a.n_sessions;
+    const int nst = static_cast<int>(a.n_steps);
+
+    auto issue = [&](uint32_t j) {
+        const uint32_t st = j & 1u;
+        const uint32_t row0 = (j % a.n_sets) * a.K + m0;
+        const uint32_t bytes = sh.n_boxes * sh.box_rows * P + cnt * 8u;
+        mbar_arrive_expect_tx(&bar[st], bytes);
+        for (uint32_t b = 0; b < sh.n_boxes; ++b)
+            tma_load_2d_hint(pay_of(st) + b * sh.box_rows * P, &tmap, 0,
+                             static_cast<int32_t>(row0 + b * sh.box_rows), &bar[st], stream_pol);
+        bulk_load_hint(out_of(st), a.outcome + row0, cnt * 4u, &bar[st], stream_pol);
+        bulk_load_hint(idx_of(st), a.idx + row0, cnt * 4u, &bar[st], stream_pol);
+        s_pending |= 1u << st;
+        s_pend_step[st] = j;
+    };
+    auto wait_stage = [&](uint32_t st, uint32_t parity) -> bool {
+        const uint64_t t0 = globaltimer_ns();
+        uint32_t spins = 0;
+        while (!mbar_try_wait(&bar[st], parity)) {
+            if ((++spins & 255u) == 0u && globaltimer_ns() - t0 > limit) return false;
+        }
+        return true;
+    };
+    auto give_up = [&](uint32_t n) {
+        latch_error(a.dev, DEV_E_TIMEOUT, n, blockIdx.x);
+        atomicExch(&a.dev->abort, 1u);
+        s_abort = 1;
+    };
+
+    if (tid == 0) {
+        mbar_init(&bar[0], 1);
+        mbar_init(&bar[1], 1);
+        fence_mbar_init();
+        s_sel = ld_volatile_u32(&a.dev->sel) & 1u;
+        s_abort = 0;
+        s_pending = 0;
+        dcount[0] = dcount[1] = 0;
+    }
+    stage_tables(tab, a.tables, a.tab_stride, 2, 0);
+    __syncthreads();
+    if (tid == 0 && cnt > 0) {
+        if (nst > 0) issue(0);
+        if (nst > 1) issue(1);
+    }
+    uint32_t sel = s_sel;
+
+    // this thread's member of the next step, prepared in phase C
+    bool pv = false;           // clean and prepared
+    uint32_t p_s = 0, p_o = 0, p_x = 0, p_odd = 0;
+    uint64_t p_rk = 0;
+    uint4 p_rec[NV];
+    uint32_t nx_s = 0, nx_o = 0;  // session / outcome of the next step's member
+
+    for (int n = -1; n < nst; ++n) {
+        const uint32_t un = static_cast<uint32_t>(n);
+        uint32_t odd = 0;
+        // ---- A: finish the clean member of step n ----
+        if (n >= 0 && mine && pv) {
+            const uint32_t y = tab[sel * a.tab_stride + p_x * 8u + p_o];
+            p_rec[0].x = y;
+            uint4 *rp = reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(p_s) * SB);
+#pragma unroll
+            for (int k = 0; k < NV; ++k) st_hint(rp + k, p_rec[k], keep_pol);
+            const size_t slot = static_cast<size_t>(un) * a.K + m0 + tid;
+            if (a.effects) {
+                uint4 e;
+                e.x = static_cast<uint32_t>(p_rk);
+                e.y = static_cast<uint32_t>(p_rk >> 32);
+                e.z = p_s;
+                e.w = y | (p_o << 16) | (sel << 24);
+                __stcs(reinterpret_cast<uint4 *>(a.effects) + slot, e);
+            }
+            if (a.state_log) {
+                uint4 *lp = reinterpret_cast<uint4 *>(a.state_log + slot * SB);
+#pragma unroll
+                for (int k = 0; k < NV; ++k) __stcs(lp + k, p_rec[k]);
+            }
+            odd = p_odd;
+        }
+        // ---- marks of cohort n + 1 (and its session / outcome for phase C) ----
+        if (n + 1 < nst && cnt > 0) {
+            const uint32_t st1 = (un + 1u) & 1u;
+            if (!wait_stage(st1, ((un + 1u) >> 1) & 1u)) give_up(un + 1u);
+            if (mine) {
+                nx_s = idx_of(st1)[tid];
+                nx_o = out_of(st1)[tid];
+                if (nx_s < N) marks[static_cast<size_t>((un + 1u) % 3u) * N + nx_s] = un + 1u;
+            }
+        }
+        if (tid == 0) dcount[(un + 1u) & 1u] = 0;
+        // ---- B: the dirty members of step n ----
+        if (n >= 0 && tid < dcount[un & 1u]) {
+            const uint32_t st = un & 1u;
+            const uint32_t t = dlist[st][tid];
+            Event<P> ev;
+            ev.s = idx_of(st)[t];
+            ev.o = out_of(st)[t];
+            read_payload_swizzled<P>(ev.pw, pay_of(st), t);
+            odd += transition<SB, P, true, true>(a, ev, tab + sel * a.tab_stride, sel, un, m0 + t, keep_pol);
+        }
+        uint32_t v = odd;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+        if ((tid & 31u) == 0) warp_odd[tid >> 5] = v;
+        __syncthreads();  // (1) step n's stores issued, counts posted, stage n & 1 free
+        if (s_abort) break;
+        unsigned long long *word = &a.dev->slot[(un + 1u) % 3u];
+        uint32_t total = 0;
+        if (tid == 0) {
+            for (uint32_t w = 0; w < (blockDim.x + 31u) / 32u; ++w) total += warp_odd[w];
+            if (!single) {
+                if (blockIdx.x == 0) a.dev->slot[(un + 2u) % 3u] = 0ull;
+                const bool skip = (n == 0 && blockIdx.x == 1 && ld_volatile_u32(&a.dev->skip_arrival) != 0u);
+                __threadfence();
+                if (!skip) red_release_add_u64(word, (1ull << 32) | total);
+            }
+        }
+        if (tid == issuer) {
+            if (n >= 0 && cnt > 0) s_pending &= ~(1u << (un & 1u));
+            if (n >= 0 && cnt > 0 && n + 2 < nst) {
+                fence_proxy_async_smem();
+                issue(un + 2u);
+            }
+        }
+        // ---- C: early work for this thread's member of step n + 1 ----
+        pv = false;
+        p_odd = 0;
+        if (n + 1 < nst && mine) {
+            const uint32_t st1 = (un + 1u) & 1u;
+            if (nx_s >= N) {
+                latch_error(a.dev, DEV_E_INDEX, un + 1u, m0 + tid);
+            } else {
+                // is this session in cohort n (whose writes are not yet visible)?
+                const bool dirty = n >= 0 && __ldcg(marks + static_cast<size_t>(un % 3u) * N + nx_s) == un;
+                if (dirty) {
+                    const uint32_t k = atomicAdd(&dcount[st1], 1u);
+                    dlist[st1][k] = static_cast<uint16_t>(tid);
+                } else {
+                    uint4 *rp = reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(nx_s) * SB);
+#pragma unroll
+                    for (int k = 0; k < NV; ++k) p_rec[k] = ld_cg_hint(rp + k, keep_pol);
+                    const uint32_t x = p_rec[0].x;
+                    if (x >= a.S || nx_o >= 8u) {
+                        latch_error(a.dev, DEV_E_STATE, un + 1u, m0 + tid);
+                    } else {
+                        uint4 pw[P / 16];
+                        read_payload_swizzled<P>(pw, pay_of(st1), tid);
+                        p_rk = route_key<P>(x, nx_o, pw);
+                        p_rec[0].y = p_rec[0].y + 1u;
+                        mix_acc<SB>(p_rec, p_rk);
+                        p_s = nx_s;
+                        p_o = nx_o;
+                        p_x = x;
+                        p_odd = static_cast<uint32_t>(p_rk & 1u);
+                        pv = true;
+                    }
+                }
+            }
+        }
+        // ---- the barrier of step n ----
+        if (tid == 0) {
+            if (single) {
+                s_sel = total > a.K / 2u ? 1u : 0u;
+            } else {
+                const uint64_t t0 = globaltimer_ns();
+                unsigned long long w;
+                uint32_t spins = 0;
+                for (;;) {
+                    w = ld_acquire_u64(word);
+                    if ((w >> 32) >= gridDim.x) break;
+                    if ((++spins & 63u) == 0u) {
+                        if (ld_volatile_u32(&a.dev->abort) != 0u) {
+                            s_abort = 1;
+                            break;
+                        }
+                        if (globaltimer_ns() - t0 > limit) {
+                            give_up(un);
+                            break;
+                        }
+                    }
+                }
+                __threadfence();
+                s_sel = (static_cast<uint32_t>(w & 0xffffffffull) > a.K / 2u) ? 1u : 0u;
+            }
+            if (n >= 0 && blockIdx.x == 0 && a.decisions && !s_abort) a.decisions[un] = s_sel;
+        }
+        __syncthreads();  // (2) decision known; dirty list of step n + 1 complete
+        if (s_abort) break;
+        if (n >= 0) sel = s_sel;
+    }
+    if (s_abort) {
+        if (tid == 0) {
+            for (uint32_t st = 0; st < 2; ++st) {
+                if (!(s_pending & (1u << st))) continue;
+                const uint32_t parity = (s_pend_step[st] >> 1) & 1u;
+                const uint64_t t0 = globaltimer_ns();
+                while (!mbar_try_wait(&bar[st], parity)) {
+                    if (globaltimer_ns() - t0 > limit) break;
+                }
+            }
+        }
+        __syncthreads();
+        return;
+    }
+    if (blockIdx.x == 0 && tid == 0) {
+        if (nst > 0) a.dev->sel = sel;
         a.dev->step = a.n_steps;
     }
 }
@@ -1066,27 +1133,15 @@ cudaError_t launch_step(const StepArgs &a, int SB, int P, int step, int sel, uin
 }
 
 namespace {
-template <int P, int D>
-const void *pipe_fn() {
-    return reinterpret_cast<const void *>(&k_chain_cta_pipe<P, D>);
-}
 template <int SB, int P, int D>
 const void *ident_fn() {
     return reinterpret_cast<const void *>(&k_chain_cta_ident<SB, P, D>);
-}
-const void *pipe_fn_rt(int P, int D) {
-    if (D == 4) return P == 32 ? pipe_fn<32, 4>() : P == 64 ? pipe_fn<64, 4>() : pipe_fn<128, 4>();
-    return P == 32 ? pipe_fn<32, 2>() : P == 64 ? pipe_fn<64, 2>() : pipe_fn<128, 2>();
 }
 const void *ident_fn_rt(int SB, int P, int D) {
     return dispatch(SB, P, [&](auto b, auto q) {
         constexpr int B = decltype(b)::value, Q = decltype(q)::value;
         return D == 4 ? ident_fn<B, Q, 4>() : D == 2 ? ident_fn<B, Q, 2>() : ident_fn<B, Q, 1>();
     });
-}
-size_t pipe_smem(uint32_t K, int P, int D, uint32_t tab_stride, uint32_t tbl_bits) {
-    const size_t Kp = (K + 3u) & ~3u, RI = 2 * D + 1, RD = D + 1, slots = size_t(1) << tbl_bits;
-    return 2 * tab_stride + RI * Kp * 4 + RD * Kp * 4 + RD * Kp * P + 2 * RD * Kp * 16 + RD * slots * 10;
 }
 size_t ident_smem(uint32_t K, int P, int D, uint32_t tab_stride) {
     const size_t Kp = (K + 3u) & ~3u, RD = D + 1;
@@ -1119,19 +1174,6 @@ cudaError_t launch_chain_cta_fast(const StepArgs &a, int SB, int P, cudaStream_t
             return cudaLaunchKernel(fn, dim3(1), dim3(threads), args, smem, s);
         }
         return cudaSuccess;
-    }
-    if (SB != 16 || K > 512u) return cudaSuccess;
-    uint32_t tbl_bits = 1;
-    while ((1u << tbl_bits) < 2u * K) ++tbl_bits;
-    for (int D : {4, 2}) {
-        const size_t smem = pipe_smem(K, P, D, a.tab_stride, tbl_bits);
-        if (smem > cap) continue;
-        const void *fn = pipe_fn_rt(P, D);
-        cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
-        if (e != cudaSuccess) return e;
-        void *args[] = {&aa, &tbl_bits};
-        *launched = true;
-        return cudaLaunchKernel(fn, dim3(1), dim3(threads), args, smem, s);
     }
     return cudaSuccess;
 }
@@ -1262,6 +1304,78 @@ cudaError_t launch_chain_grid_tma(const StepArgs &a, int SB, int P, int grid, ui
     TmaShape shc = sh;
     void *args[] = {&map, &aa, &shc};
     return cudaLaunchCooperativeKernel(grid_tma_fn(SB, P), dim3(grid), dim3(threads), args, smem, s);
+}
+
+static const void *split_fn(int SB, int P) {
+    return dispatch(SB, P, [](auto b, auto q) {
+        return reinterpret_cast<const void *>(&k_chain_split<decltype(b)::value, decltype(q)::value>);
+    });
+}
+
+bool chain_split_plan(int SB, int P, uint32_t K, uint32_t tab_stride, int *grid, uint32_t *threads, size_t *smem,
+                      void *shape_out) {
+    if (K == 0 || K % 8u != 0u || !encode_fn()) return false;
+    int dev = 0, sms = 0, max_optin = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return false;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return false;
+    if (cudaDeviceGetAttribute(&max_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+        return false;
+    TmaShape sh;
+    if (K <= 512u) {
+        sh.chunk = K;  // one CTA
+    } else {
+        const uint32_t per = (K + static_cast<uint32_t>(sms) - 1u) / static_cast<uint32_t>(sms);
+        sh.chunk = (per + 7u) & ~7u;
+        if (sh.chunk > 512u) return false;
+    }
+    const uint32_t g = (K + sh.chunk - 1u) / sh.chunk;
+    sh.n_boxes = (sh.chunk + 255u) / 256u;
+    sh.box_rows = (((sh.chunk + sh.n_boxes - 1u) / sh.n_boxes) + 7u) & ~7u;
+    sh.stage_pay = ((sh.n_boxes * sh.box_rows * static_cast<uint32_t>(P)) + 1023u) & ~1023u;
+    sh.stage_words = (sh.chunk + 3u) & ~3u;
+    const size_t bytes = tma_smem_bytes(sh, tab_stride);
+    if (bytes + 4096 > static_cast<size_t>(max_optin)) return false;
+    const void *fn = split_fn(SB, P);
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes)) !=
+        cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    const uint32_t thr = ((sh.chunk + 31u) / 32u) * 32u;
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, static_cast<int>(thr), bytes) != cudaSuccess ||
+        per_sm < 1 || static_cast<long long>(per_sm) * sms < g)
+        return false;
+    *grid = static_cast<int>(g);
+    *threads = thr;
+    *smem = bytes;
+    *static_cast<TmaShape *>(shape_out) = sh;
+    return true;
+}
+
+cudaError_t launch_chain_split(const StepArgs &a, int SB, int P, int grid, uint32_t threads, size_t smem,
+                               const void *shape, uint32_t *marks, cudaStream_t s) {
+    const TmaShape &sh = *static_cast<const TmaShape *>(shape);
+    EncodeTiled enc = encode_fn();
+    if (!enc) return cudaErrorNotSupported;
+    alignas(64) CUtensorMap map;
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(P), static_cast<cuuint64_t>(a.n_sets) * a.K};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(P)};
+    const cuuint32_t box[2] = {static_cast<cuuint32_t>(P), sh.box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUtensorMapSwizzle swz = P == 128 ? CU_TENSOR_MAP_SWIZZLE_128B
+                                   : P == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                             : CU_TENSOR_MAP_SWIZZLE_32B;
+    CUresult r = enc(&map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t *>(a.payload), dims, strides, box,
+                     estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    StepArgs aa = a;
+    TmaShape shc = sh;
+    uint32_t *mk = marks;
+    void *args[] = {&map, &aa, &shc, &mk};
+    if (grid == 1) return cudaLaunchKernel(split_fn(SB, P), dim3(1), dim3(threads), args, smem, s);
+    return cudaLaunchCooperativeKernel(split_fn(SB, P), dim3(grid), dim3(threads), args, smem, s);
 }
 
 cudaError_t launch_empty_cohorts(const StepArgs &a, cudaStream_t s) {

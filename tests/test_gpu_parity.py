@@ -173,14 +173,16 @@ def test_launch_floor_probes_run(g, rc):
         rc.rc_free(ctx)
 
 
-@pytest.mark.parametrize("tma", [True, False])
+@pytest.mark.parametrize("kernel", ["split", "tma", "plain"])
 @pytest.mark.parametrize("SB,P", [(16, 32), (16, 64), (64, 128), (64, 32)])
-@pytest.mark.parametrize("K,N,identity", [(1032, 5000, False), (4104, 9001, False), (2048, 2048, True),
-                                          (65536, 70000, False)])
-def test_persistent_grid_kernels(g, rc, monkeypatch, tma, SB, P, K, N, identity):
-    """The cooperative persistent kernels: the TMA-fed one (K a multiple of 8)
-    and the plain one, on member counts that do not split evenly over SMs."""
-    monkeypatch.setenv("RC_NO_TMA", "0" if tma else "1")
+@pytest.mark.parametrize("K,N,identity", [(1032, 5000, False), (4104, 9001, False), (4104, 4200, False),
+                                          (2048, 2048, True), (65536, 70000, False), (65536, 1 << 20, False)])
+def test_persistent_grid_kernels(g, rc, monkeypatch, kernel, SB, P, K, N, identity):
+    """The cooperative persistent kernels: split-phase (explicit sessions, K a
+    multiple of 8), TMA-fed and plain, on member counts that do not split
+    evenly over SMs, with sessions recurring from step to step (N near K)."""
+    monkeypatch.setenv("RC_NO_SPLIT", "0" if kernel == "split" else "1")
+    monkeypatch.setenv("RC_NO_TMA", "1" if kernel == "plain" else "0")
     S = 256 if SB == 64 else 64
     tables, state0, outc, pay, idx = _inputs(50 + K % 11, K, S, SB, P, 3, N=None if identity else N)
     n = 5
@@ -190,9 +192,11 @@ def test_persistent_grid_kernels(g, rc, monkeypatch, tma, SB, P, K, N, identity)
 
 
 @pytest.mark.parametrize("tma", [True, False])
-def test_grid_barrier_wait_is_bounded_both_kernels(g, rc, monkeypatch, tma):
+@pytest.mark.parametrize("split", [True, False])
+def test_grid_barrier_wait_is_bounded_both_kernels(g, rc, monkeypatch, tma, split):
     import torch
     monkeypatch.setenv("RC_NO_TMA", "0" if tma else "1")
+    monkeypatch.setenv("RC_NO_SPLIT", "0" if split else "1")
     K, S, SB, P, n = 8192, 16, 16, 64, 4
     tables, state0, outc, pay, idx = _inputs(19, K, S, SB, P, 2, N=9000)
     ctx = rc.rc_init(S, tables, SB, P, K, 9000, torch.cuda.current_stream())
@@ -215,14 +219,15 @@ def test_grid_barrier_wait_is_bounded_both_kernels(g, rc, monkeypatch, tma):
         rc.rc_free(ctx)
 
 
-@pytest.mark.parametrize("pipe", [True, False])
+@pytest.mark.parametrize("split", [True, False])
 @pytest.mark.parametrize("P", [32, 64, 128])
-@pytest.mark.parametrize("K,N", [(8, 9), (64, 67), (64, 128), (256, 259), (256, 512), (500, 1000), (512, 513)])
-def test_single_cta_pipeline_repeated_sessions(g, rc, monkeypatch, pipe, P, K, N):
+@pytest.mark.parametrize("K,N", [(8, 9), (64, 67), (64, 128), (256, 259), (256, 512), (496, 1000), (512, 513),
+                                 (100, 300)])
+def test_single_cta_repeated_sessions(g, rc, monkeypatch, split, P, K, N):
     """Sessions that recur in consecutive steps at other member positions: the
-    pipelined kernel must take their records from the steps that just wrote
-    them, not from its early copies."""
-    monkeypatch.setenv("RC_NO_PIPE", "0" if pipe else "1")
+    split-phase chain must finish them after the step that wrote them, not
+    from records read early."""
+    monkeypatch.setenv("RC_NO_SPLIT", "0" if split else "1")
     tables, state0, outc, pay, idx = _inputs(60 + K % 13 + P, K, 64, 16, P, 40, N=N)
     n = 40
     want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=1)
