@@ -188,7 +188,7 @@ def test_persistent_grid_kernels(g, rc, monkeypatch, kernel, SB, P, K, N, identi
     n = 5
     want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=1)
     got = g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K, sel0=1)
-    g.assert_same(got, want, f"grid tma={tma} K={K} SB={SB} P={P}")
+    g.assert_same(got, want, f"grid {kernel} K={K} N={N} SB={SB} P={P}")
 
 
 @pytest.mark.parametrize("tma", [True, False])
