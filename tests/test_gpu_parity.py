@@ -232,7 +232,7 @@ def test_single_cta_repeated_sessions(g, rc, monkeypatch, split, P, K, N):
     n = 40
     want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=1)
     got = g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K, sel0=1)
-    g.assert_same(got, want, f"pipe={pipe} K={K} N={N} P={P}")
+    g.assert_same(got, want, f"split={split} K={K} N={N} P={P}")
 
 
 @pytest.mark.parametrize("pipe", [True, False])
