@@ -89,7 +89,7 @@ struct rc_ctx {
     uint32_t last_launches = 0;
     bool no_tma = false;   // RC_NO_TMA=1 in the environment selects the plain grid kernel
     bool no_pipe = false;   // RC_NO_PIPE=1 selects the plain single-CTA kernel
-    bool no_split = false;  // RC_NO_SPLIT=1 turns the split-phase chain off
+    bool use_split = false;  // RC_SPLIT=1 selects the split-phase chain (slower on GB300 so far)
     Buf marks;              // split-phase cohort marks (3 * n_sessions words)
     long long *trace = nullptr;
     uint64_t trace_entries = 0;
@@ -375,7 +375,7 @@ int run_cond(rc_ctx *c, const rc::StepArgs &a) {
 
 // ---- device resident: persistent kernel ------------------------------------
 int run_persist(rc_ctx *c, const rc::StepArgs &a) {
-    if (a.idx && !c->no_split) {
+    if (a.idx && c->use_split) {
         int grid = 0;
         uint32_t threads = 0;
         size_t smem = 0;
@@ -396,8 +396,11 @@ int run_persist(rc_ctx *c, const rc::StepArgs &a) {
     if (a.K <= 1024u) {
         bool launched = false;
         if (!c->no_pipe) RC_CUDA(c, rc::launch_chain_cta_fast(a, c->SB, c->P, c->stream, &launched));
-        if (!launched) RC_CUDA(c, rc::launch_chain_cta(a, c->SB, c->P, c->stream));
-        return RC_OK;
+        if (launched) return RC_OK;
+        if (a.K <= 512u) {
+            RC_CUDA(c, rc::launch_chain_cta(a, c->SB, c->P, c->stream));
+            return RC_OK;
+        }
     }
     if (!c->coop) return fail(c, RC_E_UNSUPPORTED, "device lacks cooperative launch");
     RC_CUDA(c, cudaMemsetAsync(c->dev->slot, 0, sizeof(c->dev->slot), c->stream));
@@ -531,8 +534,8 @@ int rc_init(rc_ctx **out, uint32_t S, const uint8_t *table, uint32_t state_bytes
         c->no_tma = v && v[0] == '1';
         const char *w = std::getenv("RC_NO_PIPE");
         c->no_pipe = w && w[0] == '1';
-        const char *x = std::getenv("RC_NO_SPLIT");
-        c->no_split = x && x[0] == '1';
+        const char *x = std::getenv("RC_SPLIT");
+        c->use_split = x && x[0] == '1';
     }
     auto bail = [&](cudaError_t e) {
         rc_free(c);

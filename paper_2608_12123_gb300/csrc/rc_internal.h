@@ -74,7 +74,7 @@ dim3 step_block(uint32_t K);
 cudaError_t launch_step(const StepArgs &a, int state_bytes, int payload_bytes, int step, int sel,
                         uint32_t epi, bool decide, cudaStream_t s);
 
-// Persistent chains.  The single-CTA form takes K <= 1024; the grid form is a
+// Persistent chains.  The single-CTA form takes K <= 512; the grid form is a
 // cooperative launch of `grid` CTAs.
 cudaError_t launch_chain_cta(const StepArgs &a, int state_bytes, int payload_bytes, cudaStream_t s);
 // Pipelined single-CTA chains (identity sessions: records in registers;

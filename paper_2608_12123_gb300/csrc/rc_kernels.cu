@@ -364,12 +364,12 @@ __global__ void __launch_bounds__(kStepThreads) k_step(StepArgs a, int step_arg,
 }
 
 // ---------------------------------------------------------------------------
-// Persistent chain, one CTA (K <= 1024): all n_steps in one launch.  The
+// Persistent chain, one CTA (K <= 512): all n_steps in one launch.  The
 // decision is reduced in shared memory and read from a register: it never
-// leaves the SM.  The next step's events are fetched before the reduction.
+// leaves the SM.  Events are fetched two steps ahead.
 // ---------------------------------------------------------------------------
 template <int SB, int P>
-__global__ void __launch_bounds__(1024) k_chain_cta(StepArgs a) {
+__global__ void __launch_bounds__(512) k_chain_cta(StepArgs a) {
     __shared__ __align__(16) uint8_t tab[2 * 256 * 8];
     __shared__ uint32_t warp_odd[2][32];
     const uint32_t tid = threadIdx.x;
@@ -378,14 +378,18 @@ __global__ void __launch_bounds__(1024) k_chain_cta(StepArgs a) {
     uint32_t sel = ld_volatile_u32(&a.dev->sel) & 1u;
     __syncthreads();
     const bool active = tid < a.K;
-    Event<P> nxt;
-    if (active && a.n_steps > 0) load_event<P>(nxt, a, 0, tid);
+    // events travel two steps ahead of their use, so a step's session index
+    // is already in a register when the step starts its record gather
+    Event<P> ev0, ev1;
+    if (active && a.n_steps > 0) load_event<P>(ev0, a, 0, tid);
+    if (active && a.n_steps > 1) load_event<P>(ev1, a, 1 % a.n_sets, tid);
     for (uint32_t n = 0; n < a.n_steps; ++n) {
         uint32_t odd = 0;
         if (active) {
-            const Event<P> ev = nxt;
+            const Event<P> ev = ev0;
+            ev0 = ev1;
+            if (n + 2u < a.n_steps) load_event<P>(ev1, a, (n + 2u) % a.n_sets, tid);
             odd = transition<SB, P, false>(a, ev, tab + sel * a.tab_stride, sel, n, tid);
-            if (n + 1u < a.n_steps) load_event<P>(nxt, a, (n + 1u) % a.n_sets, tid);
         }
         const uint32_t ball = __ballot_sync(0xffffffffu, odd);
         if ((tid & 31u) == 0) warp_odd[n & 1u][tid >> 5] = __popc(ball);

@@ -181,7 +181,7 @@ def test_persistent_grid_kernels(g, rc, monkeypatch, kernel, SB, P, K, N, identi
     """The cooperative persistent kernels: split-phase (explicit sessions, K a
     multiple of 8), TMA-fed and plain, on member counts that do not split
     evenly over SMs, with sessions recurring from step to step (N near K)."""
-    monkeypatch.setenv("RC_NO_SPLIT", "0" if kernel == "split" else "1")
+    monkeypatch.setenv("RC_SPLIT", "1" if kernel == "split" else "0")
     monkeypatch.setenv("RC_NO_TMA", "1" if kernel == "plain" else "0")
     S = 256 if SB == 64 else 64
     tables, state0, outc, pay, idx = _inputs(50 + K % 11, K, S, SB, P, 3, N=None if identity else N)
@@ -196,7 +196,7 @@ def test_persistent_grid_kernels(g, rc, monkeypatch, kernel, SB, P, K, N, identi
 def test_grid_barrier_wait_is_bounded_both_kernels(g, rc, monkeypatch, tma, split):
     import torch
     monkeypatch.setenv("RC_NO_TMA", "0" if tma else "1")
-    monkeypatch.setenv("RC_NO_SPLIT", "0" if split else "1")
+    monkeypatch.setenv("RC_SPLIT", "1" if split else "0")
     K, S, SB, P, n = 8192, 16, 16, 64, 4
     tables, state0, outc, pay, idx = _inputs(19, K, S, SB, P, 2, N=9000)
     ctx = rc.rc_init(S, tables, SB, P, K, 9000, torch.cuda.current_stream())
@@ -227,7 +227,7 @@ def test_single_cta_repeated_sessions(g, rc, monkeypatch, split, P, K, N):
     """Sessions that recur in consecutive steps at other member positions: the
     split-phase chain must finish them after the step that wrote them, not
     from records read early."""
-    monkeypatch.setenv("RC_NO_SPLIT", "0" if split else "1")
+    monkeypatch.setenv("RC_SPLIT", "1" if split else "0")
     tables, state0, outc, pay, idx = _inputs(60 + K % 13 + P, K, 64, 16, P, 40, N=N)
     n = 40
     want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=1)
