@@ -65,6 +65,7 @@ extern "C" {
 #define RC_E_UNSUPPORTED (-6) /* shape or mechanism not available on this device */
 #define RC_E_INDEX (-7)       /* a kernel saw session_idx >= n_sessions (latched) */
 #define RC_E_NOMEM (-8)       /* a device or host allocation failed */
+#define RC_E_SIZE (-9)        /* larger than the fixed scratch of rc_cohort_step_noalloc allows */
 
 typedef struct rc_ctx rc_ctx;
 
@@ -193,6 +194,32 @@ int rc_set_trace(rc_ctx *ctx, void *device_buf, uint64_t bytes);
    cooperative persistent launch skips its first barrier arrival, so the other
    CTAs' bounded waits run out and RC_E_TIMEOUT is latched. */
 int rc_debug_skip_arrival(rc_ctx *ctx, uint32_t armed);
+
+/* One cohort step that allocates nothing, for callers that cannot call
+ * cudaMalloc: a serving process whose device memory is owned by another
+ * allocator, or code that must not allocate (and so must not synchronise the
+ * device) once it is running.  There is no counterpart in the paper; the
+ * arithmetic is exactly that of rc_cohort_step.
+ *   tables: DEVICE pointer to uint8 [2][S][8] (body A then B), 16-byte
+ *     aligned, every entry < S; S a power of two in [2, 256].
+ *   state (device, n_sessions records), events (device buffers, cohort 0
+ *     used), effects_out (device, K x 16 bytes, or NULL) as for rc_cohort_step.
+ *   flag: device uint32; read as this step's route body (0 = A, else B) and
+ *     overwritten with the step's decision, so consecutive calls chain on the
+ *     device without a host round trip.
+ *   status_out: device uint32 or NULL; receives 0 or the positive code of the
+ *     first bad member (4: state >= S or outcome >= 8, 7: index >= n_sessions).
+ * Its only scratch is a fixed array in the library's device code (16.6 KB on
+ * every GPU that loads the library, held until exit): up to 4,096 CTAs, so
+ * K <= 1,048,576; a larger K returns RC_E_SIZE and launches nothing.  The
+ * first call on a device resolves the array's device address (make that
+ * first call before any stream capture).  Every call shares the array and it
+ * keeps the previous call's contents: each call clears what must start at
+ * zero, and calls that overlap on the GPU race.  Asynchronous on cuda_stream;
+ * returns RC_OK, RC_E_INVAL, RC_E_SIZE or RC_E_CUDA. */
+int rc_cohort_step_noalloc(const uint8_t *tables, uint32_t S, uint32_t state_bytes, uint32_t payload_bytes,
+                           void *state, uint64_t n_sessions, const rc_events *events, uint32_t K,
+                           uint32_t *flag, void *effects_out, uint32_t *status_out, void *cuda_stream);
 
 /* ------------------------------------------------------------------------ */
 /* Online cohort former (host).  Section 9.1 (online runtime queueing events

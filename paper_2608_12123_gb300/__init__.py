@@ -27,6 +27,7 @@ RC_E_TIMEOUT = -5
 RC_E_UNSUPPORTED = -6
 RC_E_INDEX = -7
 RC_E_NOMEM = -8
+RC_E_SIZE = -9
 
 RC_MECH_HOST_RT = 0
 RC_MECH_RESIDENT_COND = 1
@@ -42,7 +43,7 @@ MECHANISMS = {"host_rt": RC_MECH_HOST_RT, "resident_cond": RC_MECH_RESIDENT_COND
 #: every symbol include/rc.h declares
 EXPORTS = ("rc_init", "rc_cohort_step", "rc_chain", "rc_free", "rc_last_error", "rc_sync",
            "rc_get_decision", "rc_set_decision", "rc_set_wait_limits", "rc_launch_floor",
-           "rc_debug_skip_arrival", "rc_last_chain_stats", "rc_set_trace", "rc_former_create", "rc_former_push", "rc_former_pop",
+           "rc_debug_skip_arrival", "rc_last_chain_stats", "rc_set_trace", "rc_cohort_step_noalloc", "rc_former_create", "rc_former_push", "rc_former_pop",
            "rc_former_push_many", "rc_former_pop_many", "rc_former_counts", "rc_former_free")
 
 
@@ -72,6 +73,7 @@ def _load():
         "rc_debug_skip_arrival": (i, [vp, u32]),
         "rc_last_chain_stats": (i, [vp, P(C.c_double), P(u32)]),
         "rc_set_trace": (i, [vp, vp, u64]),
+        "rc_cohort_step_noalloc": (i, [vp, u32, u32, u32, vp, u64, P(rc_events), u32, vp, vp, vp, vp]),
         "rc_former_create": (i, [P(vp), u32, u32, i64]),
         "rc_former_push": (i, [vp, i64, u32, u32, i64]),
         "rc_former_pop": (i, [vp, vp, P(i64), P(u32)]),
@@ -221,6 +223,20 @@ def rc_set_trace(ctx, buf, nbytes=None):
     if nbytes is None:
         nbytes = buf.numel() * buf.element_size()
     return _check(ctx, _lib.rc_set_trace(ctx.handle, _ptr(buf), int(nbytes)))
+
+
+def rc_cohort_step_noalloc(tables, S, state_bytes, payload_bytes, state, n_sessions, events, K, flag,
+                           effects=None, status=None, cuda_stream=None):
+    """The allocation-free cohort step (see include/rc.h): every buffer is the
+    caller's device memory; returns nothing, raises RcError on a rejected call."""
+    stream = None
+    if cuda_stream is not None:
+        stream = cuda_stream if isinstance(cuda_stream, int) else int(cuda_stream.cuda_stream)
+    rc = _lib.rc_cohort_step_noalloc(_ptr(tables), S, state_bytes, payload_bytes, _ptr(state), int(n_sessions),
+                                     C.byref(events), K, _ptr(flag), _ptr(effects), _ptr(status), stream)
+    if rc != RC_OK:
+        raise RcError(rc, "rc_cohort_step_noalloc rejected the call" +
+                      (" (K beyond its fixed scratch)" if rc == RC_E_SIZE else ""))
 
 
 def rc_debug_skip_arrival(ctx, armed=True):

@@ -15,8 +15,11 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <cstring>
+#include <mutex>
 #include <type_traits>
 
+#include "rc.h"
 #include "rc_internal.h"
 
 namespace rc {
@@ -1392,4 +1395,135 @@ const void *launcher_kernel() { return reinterpret_cast<const void *>(&k_launch_
 const void *empty_kernel() { return reinterpret_cast<const void *>(&k_empty); }
 const void *countdown_kernel() { return reinterpret_cast<const void *>(&k_countdown); }
 
+// ---------------------------------------------------------------------------
+// Allocation-free cohort step (rc_cohort_step_noalloc in include/rc.h).
+//
+// For callers that must not allocate device memory (the allocator belongs to
+// someone else, or allocation is not allowed once the process is serving).
+// The only scratch is a file-scope device array: an error latch and a
+// last-CTA ticket (a DevBlock) plus one odd count per CTA, summed by the last
+// CTA in CTA order.  The array is shared by every call in the process and
+// keeps the previous call's contents: the entry point clears the latch words
+// on the stream before each launch, and calls that overlap on the GPU race.
+// ---------------------------------------------------------------------------
+namespace {
+
+constexpr uint32_t kNoAllocMaxCtas = 4096;  // at most 4096 * 256 = 1,048,576 members per call
+
+struct NoAllocScratch {
+    DevBlock dev;                       // error latch, ticket (256 bytes)
+    uint32_t partial[kNoAllocMaxCtas];  // odd count of each CTA
+};
+
+static __device__ __align__(256) NoAllocScratch g_noalloc_scratch;
+
+template <int SB, int P>
+__global__ void __launch_bounds__(kStepThreads) k_step_noalloc(StepArgs a, uint32_t *flag, uint32_t *status,
+                                                              NoAllocScratch *scr) {
+    __shared__ __align__(16) uint8_t tab[256 * 8];
+    __shared__ uint32_t warp_odd[kStepThreads / 32];
+    __shared__ uint32_t s_sel;
+    const uint32_t tid = threadIdx.x;
+    if (tid == 0) s_sel = ld_volatile_u32(flag) & 1u;
+    __syncthreads();
+    const uint32_t sel = s_sel;
+    stage_tables(tab, a.tables, a.tab_stride, 1, sel);
+    __syncthreads();
+    const uint32_t m = blockIdx.x * blockDim.x + tid;
+    uint32_t odd = 0;
+    if (m < a.K) {
+        Event<P> ev;
+        load_event<P>(ev, a, 0, m);
+        odd = transition<SB, P, false>(a, ev, tab, sel, 0, m);
+    }
+    const uint32_t ball = __ballot_sync(0xffffffffu, odd);
+    if ((tid & 31u) == 0) warp_odd[tid >> 5] = __popc(ball);
+    __syncthreads();
+    if (tid != 0) return;
+    uint32_t c = 0;
+    for (uint32_t w = 0; w < (blockDim.x + 31u) / 32u; ++w) c += warp_odd[w];
+    scr->partial[blockIdx.x] = c;
+    __threadfence();
+    const uint32_t ticket = atomicAdd(&scr->dev.ticket, 1u);
+    if (ticket != gridDim.x - 1) return;
+    __threadfence();
+    uint32_t total = 0;
+    for (uint32_t b = 0; b < gridDim.x; ++b) total += ld_volatile_u32(&scr->partial[b]);
+    scr->dev.ticket = 0u;
+    *flag = total > a.K / 2u ? 1u : 0u;
+    if (status) *status = ld_volatile_u32(&scr->dev.err);
+}
+
+}  // namespace
+
+namespace {
+std::mutex g_noalloc_mu;
+void *g_noalloc_addr[64];  // device address of g_noalloc_scratch, per device (set-up on first call)
+}  // namespace
+
 }  // namespace rc
+
+extern "C" int rc_cohort_step_noalloc(const uint8_t *tables, uint32_t S, uint32_t state_bytes,
+                                      uint32_t payload_bytes, void *state, uint64_t n_sessions,
+                                      const rc_events *events, uint32_t K, uint32_t *flag, void *effects_out,
+                                      uint32_t *status_out, void *cuda_stream) {
+    using namespace rc;
+    auto a16 = [](const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
+    if (!tables || !a16(tables) || S < 2 || S > 256 || (S & (S - 1)) != 0) return RC_E_INVAL;
+    if ((state_bytes != 16 && state_bytes != 64) || (payload_bytes != 32 && payload_bytes != 64 &&
+                                                     payload_bytes != 128))
+        return RC_E_INVAL;
+    if (!state || !a16(state) || n_sessions < 1 || n_sessions > 0xffffffffull) return RC_E_INVAL;
+    if (!flag || (reinterpret_cast<uintptr_t>(flag) & 3u) != 0 || !events || events->payload_bytes != payload_bytes)
+        return RC_E_INVAL;
+    if (!a16(effects_out) || (reinterpret_cast<uintptr_t>(status_out) & 3u) != 0) return RC_E_INVAL;
+    // the scratch array holds one count per CTA: larger cohorts do not fit
+    if (K > kNoAllocMaxCtas * static_cast<uint32_t>(kStepThreads)) return RC_E_SIZE;
+    if (K > 0 && (!events->outcome || !events->payload || !a16(events->outcome) || !a16(events->payload) ||
+                  !a16(events->session_idx)))
+        return RC_E_INVAL;
+    cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return RC_E_CUDA;
+    void *scr = nullptr;
+    {
+        std::lock_guard<std::mutex> lock(g_noalloc_mu);
+        if (!g_noalloc_addr[dev]) {
+            // set-up, once per device, with that device current: the host-side
+            // name of a __device__ array is not its device address
+            void *p = nullptr;
+            if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return RC_E_CUDA;
+            g_noalloc_addr[dev] = p;
+        }
+        scr = g_noalloc_addr[dev];
+    }
+    NoAllocScratch *ns = static_cast<NoAllocScratch *>(scr);
+    // the latch and the ticket must start at zero; the array keeps the last call's contents
+    if (cudaMemsetAsync(&ns->dev, 0, sizeof(DevBlock), stream) != cudaSuccess) return RC_E_CUDA;
+    if (K == 0) {
+        if (cudaMemsetAsync(flag, 0, sizeof(uint32_t), stream) != cudaSuccess) return RC_E_CUDA;
+        if (status_out && cudaMemsetAsync(status_out, 0, sizeof(uint32_t), stream) != cudaSuccess) return RC_E_CUDA;
+        return RC_OK;
+    }
+    StepArgs a;
+    std::memset(&a, 0, sizeof(a));
+    a.state = static_cast<uint8_t *>(state);
+    a.n_sessions = n_sessions;
+    a.outcome = events->outcome;
+    a.payload = events->payload;
+    a.idx = events->session_idx;
+    a.n_sets = 1;
+    a.K = K;
+    a.tables = tables;
+    a.S = S;
+    a.tab_stride = S * 8u;
+    a.effects = static_cast<uint8_t *>(effects_out);
+    a.n_steps = 1;
+    a.dev = &ns->dev;
+    const void *fn = dispatch(static_cast<int>(state_bytes), static_cast<int>(payload_bytes), [](auto b, auto q) {
+        return reinterpret_cast<const void *>(&k_step_noalloc<decltype(b)::value, decltype(q)::value>);
+    });
+    void *args[] = {&a, &flag, &status_out, &ns};
+    if (cudaLaunchKernel(fn, step_grid(K), step_block(K), args, 0, stream) != cudaSuccess) return RC_E_CUDA;
+    return RC_OK;
+}
