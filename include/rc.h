@@ -183,11 +183,11 @@ int rc_launch_floor(rc_ctx *ctx, int kind, uint32_t reps, double *us_out);
    graph launched). */
 int rc_last_chain_stats(rc_ctx *ctx, double *device_ms_out, uint32_t *kernel_launches_out);
 
-/* Profiling aid: with a device buffer of at least 12 * n_steps int64 words
-   set, the TMA-fed persistent grid kernel records, for its first and its
-   last CTA, six SM clock readings (clock64) per step: step start, events
-   ready, members done, barrier arrival, next copies issued, barrier passed.
-   Layout [2][n_steps][6].  NULL (the default) turns it off. */
+/* Profiling aid: with a device buffer of at least 16 * n_steps int64 words
+   set, the persistent grid kernels record, for their first and last CTA, up
+   to eight SM clock readings (clock64) per step at their phase boundaries
+   (layout [2][n_steps][8]; the phases are listed beside each kernel in the
+   library source).  NULL (the default) turns it off. */
 int rc_set_trace(rc_ctx *ctx, void *device_buf, uint64_t bytes);
 
 /* Test hook (device-side bounded-wait check): when armed, CTA 1 of the next

@@ -90,6 +90,8 @@ struct rc_ctx {
     bool no_tma = false;   // RC_NO_TMA=1 in the environment selects the plain grid kernel
     bool no_pipe = false;   // RC_NO_PIPE=1 selects the plain single-CTA kernel
     bool use_split = false;  // RC_SPLIT=1 selects the split-phase chain (slower on GB300 so far)
+    bool use_owned = false;  // RC_OWNED=1 selects the session-owned chain
+    Buf route_buf;           // session-owned chain: routed member lists
     Buf marks;              // split-phase cohort marks (3 * n_sessions words)
     long long *trace = nullptr;
     uint64_t trace_entries = 0;
@@ -225,7 +227,7 @@ int resolve(rc_ctx *c, void *state, const rc_events *ev, uint32_t K, uint32_t n_
     a.n_steps = n_steps;
     a.dev = c->dev;
     a.h_while = 0;
-    a.trace = (c->trace && c->trace_entries >= 12ull * n_steps) ? c->trace : nullptr;
+    a.trace = (c->trace && c->trace_entries >= 16ull * n_steps) ? c->trace : nullptr;
     const size_t n_ev = static_cast<size_t>(n_sets) * K;
     a.outcome = ev->outcome;
     a.payload = ev->payload;
@@ -375,6 +377,26 @@ int run_cond(rc_ctx *c, const rc::StepArgs &a) {
 
 // ---- device resident: persistent kernel ------------------------------------
 int run_persist(rc_ctx *c, const rc::StepArgs &a) {
+    if (a.idx && c->use_owned && c->coop) {
+        int grid = 0;
+        uint32_t threads = 0;
+        size_t smem = 0;
+        alignas(8) unsigned char shape[32];
+        if (rc::chain_owned_plan(c->SB, c->P, a.K, c->n_sessions, c->tab_stride, &grid, &threads, &smem, shape)) {
+            const size_t nev = static_cast<size_t>(a.n_sets) * a.K;
+            int rc = ensure(c, c->route_buf, nev * 12 + static_cast<size_t>(a.n_sets) * (grid + 1) * 4 + 64);
+            if (rc != RC_OK) return rc;
+            uint32_t *pm = static_cast<uint32_t *>(c->route_buf.p);
+            uint32_t *ps = pm + nev, *po = ps + nev, *off = po + nev;
+            RC_CUDA(c, cudaMemsetAsync(c->dev->slot4, 0, sizeof(c->dev->slot4), c->stream));
+            RC_CUDA(c, cudaMemsetAsync(&c->dev->abort, 0, sizeof(uint32_t), c->stream));
+            RC_CUDA(c, rc::launch_route(a, shape, pm, ps, po, off, c->stream));
+            RC_CUDA(c, rc::launch_chain_owned(a, c->SB, c->P, grid, threads, smem, shape, pm, ps, po, off,
+                                              c->stream));
+            RC_CUDA(c, cudaMemsetAsync(&c->dev->skip_arrival, 0, sizeof(uint32_t), c->stream));
+            return RC_OK;
+        }
+    }
     if (a.idx && c->use_split) {
         int grid = 0;
         uint32_t threads = 0;
@@ -536,6 +558,8 @@ int rc_init(rc_ctx **out, uint32_t S, const uint8_t *table, uint32_t state_bytes
         c->no_pipe = w && w[0] == '1';
         const char *x = std::getenv("RC_SPLIT");
         c->use_split = x && x[0] == '1';
+        const char *y = std::getenv("RC_OWNED");
+        c->use_owned = y && y[0] == '1';
     }
     auto bail = [&](cudaError_t e) {
         rc_free(c);
@@ -639,7 +663,7 @@ int rc_free(rc_ctx *c) {
     c->cond.reset();
     c->floor.reset();
     c->nested.reset();
-    for (Buf *b : {&c->st_outcome, &c->st_payload, &c->st_idx, &c->st_dec, &c->st_eff, &c->st_log, &c->marks})
+    for (Buf *b : {&c->st_outcome, &c->st_payload, &c->st_idx, &c->st_dec, &c->st_eff, &c->st_log, &c->marks, &c->route_buf})
         if (b->p) cudaFree(b->p);
     if (c->d_tables) cudaFree(c->d_tables);
     if (c->dev) cudaFree(c->dev);

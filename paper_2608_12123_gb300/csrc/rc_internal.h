@@ -24,6 +24,8 @@ struct alignas(256) DevBlock {
     uint64_t wait_ns;       // device spin-wait limit (ns of %globaltimer)
     unsigned long long slot[3];  // grid-barrier words of the persistent grid kernel
     uint32_t countdown;     // launch-floor probe: WHILE iterations left
+    uint32_t pad1;
+    unsigned long long slot4[4];  // monotonic count words of the session-owned chain
 };
 
 // Everything a step kernel needs.  Event arrays hold n_sets cohorts of K;
@@ -100,6 +102,17 @@ bool chain_split_plan(int state_bytes, int payload_bytes, uint32_t K, uint32_t t
                       uint32_t *threads, size_t *smem, void *shape_out);
 cudaError_t launch_chain_split(const StepArgs &a, int state_bytes, int payload_bytes, int grid, uint32_t threads,
                                size_t smem, const void *shape, uint32_t *marks, cudaStream_t s);
+
+// Session-owned persistent chain: k_route groups each cohort's members by the
+// CTA owning their session (perm_* : n_sets * K words each, off : n_sets *
+// (G + 1) words), then k_chain_owned runs the chain.
+bool chain_owned_plan(int state_bytes, int payload_bytes, uint32_t K, uint64_t n_sessions, uint32_t tab_stride,
+                      int *grid, uint32_t *threads, size_t *smem, void *shape_out);
+cudaError_t launch_route(const StepArgs &a, const void *shape, uint32_t *perm_m, uint32_t *perm_s, uint32_t *perm_o,
+                         uint32_t *off, cudaStream_t s);
+cudaError_t launch_chain_owned(const StepArgs &a, int state_bytes, int payload_bytes, int grid, uint32_t threads,
+                               size_t smem, const void *shape, const uint32_t *perm_m, const uint32_t *perm_s,
+                               const uint32_t *perm_o, const uint32_t *off, cudaStream_t s);
 
 // Writes decisions[0..n) = 0 and sel = 0 (an empty cohort decides 0).
 cudaError_t launch_empty_cohorts(const StepArgs &a, cudaStream_t s);

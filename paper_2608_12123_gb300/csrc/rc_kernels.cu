@@ -658,9 +658,9 @@ __global__ void __launch_bounds__(512, 1)
     const uint64_t stream_pol = policy_evict_first();
     const uint64_t keep_pol = policy_evict_last();
     const uint32_t issuer = blockDim.x > 32u ? 32u : 0u;  // lane 0 of warp 1 issues the copies
-    // profiling: thread 0 of the first and last CTA records six phase clocks per step
+    // profiling: thread 0 of the first and last CTA records phase clocks per step
     long long *trace = (a.trace && tid == 0 && (blockIdx.x == 0 || blockIdx.x == gridDim.x - 1))
-                           ? a.trace + (blockIdx.x == 0 ? 0 : static_cast<size_t>(a.n_steps) * 6)
+                           ? a.trace + (blockIdx.x == 0 ? 0 : static_cast<size_t>(a.n_steps) * 8)
                            : nullptr;
 
     // thread 0 issues the copies of step j into stage j & 1
@@ -705,7 +705,7 @@ __global__ void __launch_bounds__(512, 1)
     for (uint32_t n = 0; n < a.n_steps; ++n) {
         const uint32_t st = n & 1u;
         uint32_t odd = 0;
-        if (trace) trace[n * 6 + 0] = clock64();
+        if (trace) trace[n * 8 + 0] = clock64();
         if (cnt > 0) {
             if (!wait_stage(st, (n >> 1) & 1u)) {
                 latch_error(a.dev, DEV_E_TIMEOUT, n, blockIdx.x);
@@ -715,7 +715,7 @@ __global__ void __launch_bounds__(512, 1)
         }
         __syncthreads();
         if (s_abort) break;
-        if (trace) trace[n * 6 + 1] = clock64();
+        if (trace) trace[n * 8 + 1] = clock64();
         for (uint32_t t = tid; t < cnt; t += blockDim.x) {
             Event<P> ev;
             ev.s = a.idx ? idx_of(st)[t] : m0 + t;
@@ -729,7 +729,7 @@ __global__ void __launch_bounds__(512, 1)
         if ((tid & 31u) == 0) warp_odd[tid >> 5] = v;
         __syncthreads();  // every thread is done with stage st and has stored this step's records
         if (tid == 0) {
-            if (trace) trace[n * 6 + 2] = clock64();
+            if (trace) trace[n * 8 + 2] = clock64();
             uint32_t c = 0;
             for (uint32_t w = 0; w < (blockDim.x + 31u) / 32u; ++w) c += warp_odd[w];
             unsigned long long *word = &a.dev->slot[n % 3u];
@@ -737,7 +737,7 @@ __global__ void __launch_bounds__(512, 1)
             __threadfence();
             const bool skip = (n == 0 && blockIdx.x == 1 && ld_volatile_u32(&a.dev->skip_arrival) != 0u);
             if (!skip) red_release_add_u64(word, (1ull << 32) | c);
-            if (trace) trace[n * 6 + 3] = clock64();
+            if (trace) trace[n * 8 + 3] = clock64();
             if (issuer == 0) {
                 if (cnt > 0) s_pending &= ~(1u << st);
                 if (cnt > 0 && n + 2u < a.n_steps) {
@@ -745,7 +745,7 @@ __global__ void __launch_bounds__(512, 1)
                     issue(n + 2u);
                 }
             }
-            if (trace) trace[n * 6 + 4] = clock64();
+            if (trace) trace[n * 8 + 4] = clock64();
             const uint64_t t0 = globaltimer_ns();
             unsigned long long w;
             uint32_t spins = 0;
@@ -766,7 +766,7 @@ __global__ void __launch_bounds__(512, 1)
                 }
             }
             __threadfence();
-            if (trace) trace[n * 6 + 5] = clock64();
+            if (trace) trace[n * 8 + 5] = clock64();
             const uint32_t d = (static_cast<uint32_t>(w & 0xffffffffull) > a.K / 2u) ? 1u : 0u;
             s_sel = d;
             if (blockIdx.x == 0 && a.decisions && !s_abort) a.decisions[n] = d;
@@ -858,6 +858,12 @@ __global__ void __launch_bounds__(512, 1)
     const uint32_t issuer = blockDim.x > 32u ? 32u : 0u;
     const uint64_t N = a.n_sessions;
     const int nst = static_cast<int>(a.n_steps);
+    long long *trace = (a.trace && tid == 0 && (blockIdx.x == 0 || blockIdx.x == gridDim.x - 1))
+                           ? a.trace + (blockIdx.x == 0 ? 0 : static_cast<size_t>(a.n_steps) * 8)
+                           : nullptr;
+    auto mark_time = [&](int n, int k) {
+        if (trace && n >= 0) trace[static_cast<size_t>(n) * 8 + k] = clock64();
+    };
 
     auto issue = [&](uint32_t j) {
         const uint32_t st = j & 1u;
@@ -913,6 +919,7 @@ __global__ void __launch_bounds__(512, 1)
     for (int n = -1; n < nst; ++n) {
         const uint32_t un = static_cast<uint32_t>(n);
         uint32_t odd = 0;
+        mark_time(n, 0);
         // ---- A: finish the clean member of step n ----
         if (n >= 0 && mine && pv) {
             const uint32_t y = tab[sel * a.tab_stride + p_x * 8u + p_o];
@@ -947,6 +954,7 @@ __global__ void __launch_bounds__(512, 1)
             }
         }
         if (tid == 0) dcount[(un + 1u) & 1u] = 0;
+        mark_time(n, 1);
         // ---- B: the dirty members of step n ----
         if (n >= 0 && tid < dcount[un & 1u]) {
             const uint32_t st = un & 1u;
@@ -957,12 +965,14 @@ __global__ void __launch_bounds__(512, 1)
             read_payload_swizzled<P>(ev.pw, pay_of(st), t);
             odd += transition<SB, P, true, true>(a, ev, tab + sel * a.tab_stride, sel, un, m0 + t, keep_pol);
         }
+        mark_time(n, 2);
         uint32_t v = odd;
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
         if ((tid & 31u) == 0) warp_odd[tid >> 5] = v;
         __syncthreads();  // (1) step n's stores issued, counts posted, stage n & 1 free
         if (s_abort) break;
+        mark_time(n, 3);
         unsigned long long *word = &a.dev->slot[(un + 1u) % 3u];
         uint32_t total = 0;
         if (tid == 0) {
@@ -973,6 +983,7 @@ __global__ void __launch_bounds__(512, 1)
                 __threadfence();
                 if (!skip) red_release_add_u64(word, (1ull << 32) | total);
             }
+            mark_time(n, 4);
         }
         if (tid == issuer) {
             if (n >= 0 && cnt > 0) s_pending &= ~(1u << (un & 1u));
@@ -1017,6 +1028,7 @@ __global__ void __launch_bounds__(512, 1)
             }
         }
         // ---- the barrier of step n ----
+        mark_time(n, 5);
         if (tid == 0) {
             if (single) {
                 s_sel = total > a.K / 2u ? 1u : 0u;
@@ -1042,8 +1054,10 @@ __global__ void __launch_bounds__(512, 1)
                 s_sel = (static_cast<uint32_t>(w & 0xffffffffull) > a.K / 2u) ? 1u : 0u;
             }
             if (n >= 0 && blockIdx.x == 0 && a.decisions && !s_abort) a.decisions[un] = s_sel;
+            mark_time(n, 6);
         }
         __syncthreads();  // (2) decision known; dirty list of step n + 1 complete
+        mark_time(n, 7);
         if (s_abort) break;
         if (n >= 0) sel = s_sel;
     }
@@ -1064,6 +1078,370 @@ __global__ void __launch_bounds__(512, 1)
     if (blockIdx.x == 0 && tid == 0) {
         if (nst > 0) a.dev->sel = sel;
         a.dev->step = a.n_steps;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Persistent chain with session ownership (explicit session indices; G CTAs,
+// CTA b owns sessions [b*per, (b+1)*per)).
+//
+// k_route groups every cohort's members by the CTA that owns their session:
+// for cohort j it writes, contiguously per owner, the member index, the
+// session and the outcome (owner b's run is [off[j][b], off[j][b+1])).
+// k_chain_owned then lets each CTA transition only its own sessions, so no
+// CTA ever reads a record another CTA writes: the state field of every owned
+// session lives in shared memory (the whole record when RES), the per-step
+// grid barrier carries nothing but the odd-key count (a relaxed atomic on a
+// monotonic word per step mod 4, no fence), and a CTA arrives for step n
+// before it waits for the decision of step n - 1, so that wait overlaps a
+// whole step of route-key work.  Iteration n:
+//   1. its payload rows (TMA-free: per-thread async copies, issued one step
+//      ahead) and run of step n are ready; (non-RES) issue the record loads;
+//   2. route key of every owned member from the state in shared memory;
+//   3. post the odd count of step n (relaxed add);
+//   4. wait for step n - 1's count: decision d_{n-1} = body of step n;
+//   5. next state y = T_d[x][o] into shared memory, record and effect out.
+// Four steps of barrier words suffice: a CTA can arrive for step k + 4 only
+// after the barrier of step k + 2 completed, that is after every CTA has
+// read the word of step k.  Waits are bounded as in the other grid kernels.
+// ---------------------------------------------------------------------------
+__global__ void k_route(const uint32_t *idx, const uint32_t *outcome, uint32_t n_sets, uint32_t K, uint64_t N,
+                        uint32_t G, uint32_t per, uint32_t *perm_m, uint32_t *perm_s, uint32_t *perm_o,
+                        uint32_t *off, DevBlock *dev) {
+    extern __shared__ uint32_t hist[];  // [G + 1]
+    const uint32_t j = blockIdx.x;
+    for (uint32_t b = threadIdx.x; b <= G; b += blockDim.x) hist[b] = 0;
+    __syncthreads();
+    const size_t e0 = static_cast<size_t>(j) * K;
+    for (uint32_t m = threadIdx.x; m < K; m += blockDim.x) {
+        const uint32_t s = idx ? idx[e0 + m] : m;
+        if (s < N) atomicAdd(&hist[s / per], 1u);
+        else latch_error(dev, DEV_E_INDEX, 0xffffffffu, m);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {  // exclusive scan (G <= a few hundred)
+        uint32_t acc = 0;
+        for (uint32_t b = 0; b < G; ++b) {
+            const uint32_t c = hist[b];
+            hist[b] = acc;
+            off[static_cast<size_t>(j) * (G + 1) + b] = acc;
+            acc += c;
+        }
+        off[static_cast<size_t>(j) * (G + 1) + G] = acc;
+    }
+    __syncthreads();
+    for (uint32_t m = threadIdx.x; m < K; m += blockDim.x) {
+        const uint32_t s = idx ? idx[e0 + m] : m;
+        if (s >= N) continue;
+        const uint32_t p = atomicAdd(&hist[s / per], 1u);
+        perm_m[e0 + p] = m;
+        perm_s[e0 + p] = s;
+        perm_o[e0 + p] = outcome[e0 + m];
+    }
+}
+
+struct OwnedShape {
+    uint32_t G;    // CTAs
+    uint32_t per;  // sessions owned per CTA
+    uint32_t res;  // records resident in shared memory
+    uint32_t pad;
+};
+
+__device__ __forceinline__ uint32_t ld_relaxed_hi(const unsigned long long *p, uint32_t *lo) {
+    unsigned long long v;
+    asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+    *lo = static_cast<uint32_t>(v);
+    return static_cast<uint32_t>(v >> 32);
+}
+
+// One routed member: index in its cohort, session, outcome; valid when this
+// thread's slot lies inside its CTA's run.
+struct Routed {
+    uint32_t m, s, o, valid;
+};
+
+template <int SB, int P, bool RES>
+__global__ void __launch_bounds__(512, 1)
+    k_chain_owned(StepArgs a, OwnedShape sh, const uint32_t *perm_m, const uint32_t *perm_s,
+                  const uint32_t *perm_o, const uint32_t *off) {
+    constexpr int NV = SB / 16;
+    constexpr uint32_t NC = P / 16;
+    extern __shared__ __align__(16) uint8_t dsm[];
+    __shared__ uint32_t warp_odd[16];
+    __shared__ uint32_t s_sel, s_abort;
+    const uint32_t tid = threadIdx.x;
+    const uint32_t T = blockDim.x;
+    const uint32_t b = blockIdx.x;
+    const uint32_t G = gridDim.x;
+    const uint32_t nst = a.n_steps;
+    const uint64_t limit = a.dev->wait_ns;
+    const uint32_t base_s = b * sh.per;
+    const uint64_t left = base_s < a.n_sessions ? a.n_sessions - base_s : 0ull;
+    const uint32_t own = left < sh.per ? static_cast<uint32_t>(left) : sh.per;
+    const size_t n_ev = static_cast<size_t>(a.n_sets) * a.K;
+    long long *trace = (a.trace && tid == 0 && (b == 0 || b == G - 1))
+                           ? a.trace + (b == 0 ? 0 : static_cast<size_t>(nst) * 8)
+                           : nullptr;
+    // shared layout: [tables][payload rows: 2 stages x T][record stage: T (not RES)][owned states or records]
+    uint8_t *tab = dsm;
+    uint4 *pay = reinterpret_cast<uint4 *>(dsm + 2 * a.tab_stride);
+    uint4 *rec_st = pay + 2ull * T * NC;
+    uint8_t *owned = reinterpret_cast<uint8_t *>(rec_st + (RES ? 0ull : static_cast<size_t>(T) * NV));
+    uint4 *owned_rec = reinterpret_cast<uint4 *>(owned);  // RES: [per][NV]
+
+    stage_tables(tab, a.tables, a.tab_stride, 2, 0);
+    for (uint32_t ls = tid; ls < own; ls += T) {
+        const uint4 *rp = reinterpret_cast<const uint4 *>(a.state + static_cast<size_t>(base_s + ls) * SB);
+        if constexpr (RES) {
+#pragma unroll
+            for (int k = 0; k < NV; ++k) owned_rec[static_cast<size_t>(ls) * NV + k] = rp[k];
+        } else {
+            owned[ls] = static_cast<uint8_t>(__ldg(reinterpret_cast<const uint32_t *>(rp)));
+        }
+    }
+    if (tid == 0) {
+        s_sel = ld_volatile_u32(&a.dev->sel) & 1u;
+        s_abort = 0;
+    }
+
+    // run of step j for this CTA (two plain loads; clamped so that no branch waits on them)
+    auto load_run = [&](uint32_t j, uint32_t &lo, uint32_t &hi) {
+        const uint32_t jj = j < nst ? j : 0u;
+        const size_t o = static_cast<size_t>(jj % a.n_sets) * (G + 1) + b;
+        lo = __ldg(off + o);
+        hi = __ldg(off + o + 1);
+        if (j >= nst) hi = lo;  // applied when the values are used
+    };
+    // this thread's entry of step j's run (clamped address, validity kept apart)
+    auto load_entry = [&](uint32_t j, uint32_t lo, uint32_t hi, Routed &r) {
+        const bool v = j < nst && tid < hi - lo;
+        size_t e = static_cast<size_t>((j < nst ? j : 0u) % a.n_sets) * a.K + lo + tid;
+        e = v ? e : 0;
+        e = e < n_ev ? e : 0;
+        r.m = __ldg(perm_m + e);
+        r.s = __ldg(perm_s + e);
+        r.o = __ldg(perm_o + e);
+        r.valid = v ? 1u : 0u;
+    };
+    auto stage_row = [&](uint32_t j, const Routed &r) {
+        if (!r.valid) return;
+        const uint4 *src =
+            reinterpret_cast<const uint4 *>(a.payload + (static_cast<size_t>(j % a.n_sets) * a.K + r.m) * P);
+        uint4 *dst = pay + static_cast<size_t>(j & 1u) * T * NC;
+#pragma unroll
+        for (uint32_t k = 0; k < NC; ++k) cp_async16(dst + pay_chunk<P>(tid, k), src + k);
+    };
+    auto stage_record = [&](const Routed &r) {
+        if constexpr (!RES) {
+            if (!r.valid) return;
+            const uint4 *rp = reinterpret_cast<const uint4 *>(a.state + static_cast<size_t>(r.s) * SB);
+#pragma unroll
+            for (int k = 0; k < NV; ++k) cp_async16(rec_st + static_cast<size_t>(tid) * NV + k, rp + k);
+        }
+    };
+    auto wait_count = [&](uint32_t k, uint32_t *low_prev) -> uint32_t {
+        const uint32_t target = (k / 4u + 1u) * G;
+        const uint64_t t0 = globaltimer_ns();
+        uint32_t spins = 0, low = 0;
+        for (;;) {
+            const uint32_t hi = ld_relaxed_hi(&a.dev->slot4[k & 3u], &low);
+            if (hi >= target) break;
+            __nanosleep(64);
+            if ((++spins & 31u) == 0u) {
+                if (ld_volatile_u32(&a.dev->abort) != 0u) {
+                    s_abort = 1;
+                    break;
+                }
+                if (globaltimer_ns() - t0 > limit) {
+                    latch_error(a.dev, DEV_E_TIMEOUT, k, b);
+                    atomicExch(&a.dev->abort, 1u);
+                    s_abort = 1;
+                    break;
+                }
+            }
+        }
+        const uint32_t total = low - low_prev[k & 3u];
+        low_prev[k & 3u] = low;
+        return total > a.K / 2u ? 1u : 0u;
+    };
+
+    // pipeline: runs three steps ahead, entries two, rows one
+    uint32_t lo0, hi0, lo1, hi1, lo2, hi2, lo3, hi3;
+    Routed r0, r1, r2;
+    load_run(0, lo0, hi0);
+    load_run(1, lo1, hi1);
+    load_run(2, lo2, hi2);
+    load_entry(0, lo0, hi0, r0);
+    load_entry(1, lo1, hi1, r1);
+    stage_row(0, r0);
+    cp_async_commit();
+    __syncthreads();
+    uint32_t sel = s_sel;
+    uint32_t low_prev[4] = {0u, 0u, 0u, 0u};
+
+    for (uint32_t n = 0; n < nst; ++n) {
+        if (trace) trace[n * 8 + 0] = clock64();
+        load_run(n + 3u, lo3, hi3);
+        load_entry(n + 2u, lo2, hi2, r2);
+        stage_record(r0);           // records of step n (the previous step's writes are done)
+        cp_async_commit();
+        stage_row(n + 1u, r1);      // rows of step n + 1
+        cp_async_commit();
+        cp_async_wait<2>();         // this thread's row of step n is here
+        if (trace) trace[n * 8 + 1] = clock64();
+        const size_t e0 = static_cast<size_t>(n % a.n_sets) * a.K;
+        const uint32_t cnt0 = hi0 - lo0;
+        uint32_t odd = 0, x = 0;
+        uint64_t rk = 0;
+        bool ok = false;
+        if (r0.valid) {
+            const uint32_t ls = r0.s - base_s;
+            x = RES ? owned_rec[static_cast<size_t>(ls) * NV].x : static_cast<uint32_t>(owned[ls]);
+            if (x >= a.S || r0.o >= 8u) {
+                latch_error(a.dev, DEV_E_STATE, n, r0.m);
+            } else {
+                const uint4 *stage = pay + static_cast<size_t>(n & 1u) * T * NC;
+                uint4 pw[NC];
+#pragma unroll
+                for (uint32_t k = 0; k < NC; ++k) pw[k] = stage[pay_chunk<P>(tid, k)];
+                rk = route_key<P>(x, r0.o, pw);
+                odd = static_cast<uint32_t>(rk & 1u);
+                ok = true;
+            }
+        }
+        // members beyond one per thread (rare): keys now, state after the decision
+        for (uint32_t p = tid + T; p < cnt0; p += T) {
+            const size_t e = e0 + lo0 + p;
+            const uint32_t s2 = __ldg(perm_s + e), m2 = __ldg(perm_m + e), o2 = __ldg(perm_o + e);
+            const uint32_t x2 = RES ? owned_rec[static_cast<size_t>(s2 - base_s) * NV].x : owned[s2 - base_s];
+            if (x2 >= a.S || o2 >= 8u) {
+                latch_error(a.dev, DEV_E_STATE, n, m2);
+                continue;
+            }
+            uint4 pw[NC];
+            const uint4 *src = reinterpret_cast<const uint4 *>(a.payload + (e0 + m2) * P);
+#pragma unroll
+            for (uint32_t k = 0; k < NC; ++k) pw[k] = __ldg(src + k);
+            odd += static_cast<uint32_t>(route_key<P>(x2, o2, pw) & 1u);
+        }
+        if (trace) trace[n * 8 + 2] = clock64();
+        uint32_t v = odd;
+#pragma unroll
+        for (int o2 = 16; o2 > 0; o2 >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o2);
+        if ((tid & 31u) == 0) warp_odd[tid >> 5] = v;
+        __syncthreads();
+        if (tid == 0) {
+            if (trace) trace[n * 8 + 3] = clock64();
+            uint32_t c = 0;
+            for (uint32_t w = 0; w < (T + 31u) / 32u; ++w) c += warp_odd[w];
+            // post step n's count (nothing else crosses CTAs), then take step n - 1's decision
+            const bool skip = (n == 0 && b == 1 && ld_volatile_u32(&a.dev->skip_arrival) != 0u);
+            if (!skip) atomicAdd(&a.dev->slot4[n & 3u], (1ull << 32) | c);
+            if (trace) trace[n * 8 + 4] = clock64();
+            if (n > 0) {
+                s_sel = wait_count(n - 1u, low_prev);
+                if (b == 0 && a.decisions && !s_abort) a.decisions[n - 1u] = s_sel;
+            }
+            if (trace) trace[n * 8 + 5] = clock64();
+        }
+        __syncthreads();
+        if (s_abort) break;
+        if (n > 0) sel = s_sel;
+        cp_async_wait<1>();  // this thread's record of step n is here
+        if (trace) trace[n * 8 + 6] = clock64();
+        // --- next state, record and effect (body chosen by the decision of step n - 1) ---
+        auto finish = [&](uint32_t s2, uint32_t m2, uint32_t o2, uint32_t x2, uint64_t rk2, uint4 (&rr)[NV]) {
+            const uint32_t y = tab[sel * a.tab_stride + x2 * 8u + o2];
+            rr[0].x = y;
+            rr[0].y = rr[0].y + 1u;
+            mix_acc<SB>(rr, rk2);
+            const uint32_t ls = s2 - base_s;
+            if constexpr (RES) {
+#pragma unroll
+                for (int k = 0; k < NV; ++k) owned_rec[static_cast<size_t>(ls) * NV + k] = rr[k];
+            } else {
+                owned[ls] = static_cast<uint8_t>(y);
+                uint4 *rp = reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(s2) * SB);
+#pragma unroll
+                for (int k = 0; k < NV; ++k) rp[k] = rr[k];
+            }
+            const size_t slot = static_cast<size_t>(n) * a.K + m2;
+            if (a.effects) {
+                uint4 e;
+                e.x = static_cast<uint32_t>(rk2);
+                e.y = static_cast<uint32_t>(rk2 >> 32);
+                e.z = s2;
+                e.w = y | (o2 << 16) | (sel << 24);
+                __stcs(reinterpret_cast<uint4 *>(a.effects) + slot, e);
+            }
+            if (a.state_log) {
+                uint4 *lp = reinterpret_cast<uint4 *>(a.state_log + slot * SB);
+#pragma unroll
+                for (int k = 0; k < NV; ++k) __stcs(lp + k, rr[k]);
+            }
+        };
+        if (ok) {
+            uint4 rr[NV];
+            if constexpr (RES) {
+#pragma unroll
+                for (int k = 0; k < NV; ++k) rr[k] = owned_rec[static_cast<size_t>(r0.s - base_s) * NV + k];
+            } else {
+#pragma unroll
+                for (int k = 0; k < NV; ++k) rr[k] = rec_st[static_cast<size_t>(tid) * NV + k];
+            }
+            finish(r0.s, r0.m, r0.o, x, rk, rr);
+        }
+        for (uint32_t p = tid + T; p < cnt0; p += T) {
+            const size_t e = e0 + lo0 + p;
+            const uint32_t s2 = __ldg(perm_s + e), m2 = __ldg(perm_m + e), o2 = __ldg(perm_o + e);
+            uint4 rr[NV];
+            uint32_t x2;
+            if constexpr (RES) {
+#pragma unroll
+                for (int k = 0; k < NV; ++k) rr[k] = owned_rec[static_cast<size_t>(s2 - base_s) * NV + k];
+                x2 = rr[0].x;
+            } else {
+                const uint4 *rp = reinterpret_cast<const uint4 *>(a.state + static_cast<size_t>(s2) * SB);
+#pragma unroll
+                for (int k = 0; k < NV; ++k) rr[k] = __ldcg(rp + k);
+                x2 = owned[s2 - base_s];
+            }
+            if (x2 >= a.S || o2 >= 8u) continue;
+            uint4 pw[NC];
+            const uint4 *src = reinterpret_cast<const uint4 *>(a.payload + (e0 + m2) * P);
+#pragma unroll
+            for (uint32_t k = 0; k < NC; ++k) pw[k] = __ldg(src + k);
+            finish(s2, m2, o2, x2, route_key<P>(x2, o2, pw), rr);
+        }
+        __syncthreads();  // owned state updated before the next step reads it; stages free
+        if (trace) trace[n * 8 + 7] = clock64();
+        lo0 = lo1;
+        hi0 = hi1;
+        r0 = r1;
+        lo1 = lo2;
+        hi1 = hi2;
+        r1 = r2;
+        lo2 = lo3;
+        hi2 = hi3;
+    }
+    cp_async_wait<0>();
+    if (tid == 0 && !s_abort && nst > 0) {
+        s_sel = wait_count(nst - 1u, low_prev);
+        if (b == 0 && !s_abort) {
+            if (a.decisions) a.decisions[nst - 1u] = s_sel;
+            a.dev->sel = s_sel;
+            a.dev->step = nst;
+        }
+    }
+    __syncthreads();
+    if constexpr (RES) {
+        if (!s_abort) {
+            for (uint32_t ls = tid; ls < own; ls += T) {
+                uint4 *rp = reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(base_s + ls) * SB);
+#pragma unroll
+                for (int k = 0; k < NV; ++k) rp[k] = owned_rec[static_cast<size_t>(ls) * NV + k];
+            }
+        }
     }
 }
 
@@ -1383,6 +1761,73 @@ cudaError_t launch_chain_split(const StepArgs &a, int SB, int P, int grid, uint3
     void *args[] = {&map, &aa, &shc, &mk};
     if (grid == 1) return cudaLaunchKernel(split_fn(SB, P), dim3(1), dim3(threads), args, smem, s);
     return cudaLaunchCooperativeKernel(split_fn(SB, P), dim3(grid), dim3(threads), args, smem, s);
+}
+
+static const void *owned_fn(int SB, int P, bool res) {
+    return dispatch(SB, P, [&](auto b, auto q) {
+        constexpr int B = decltype(b)::value, Q = decltype(q)::value;
+        return res ? reinterpret_cast<const void *>(&k_chain_owned<B, Q, true>)
+                   : reinterpret_cast<const void *>(&k_chain_owned<B, Q, false>);
+    });
+}
+
+bool chain_owned_plan(int SB, int P, uint32_t K, uint64_t N, uint32_t tab_stride, int *grid, uint32_t *threads,
+                      size_t *smem, void *shape_out) {
+    if (K == 0) return false;
+    int dev = 0, sms = 0, max_optin = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return false;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return false;
+    if (cudaDeviceGetAttribute(&max_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+        return false;
+    OwnedShape sh;
+    sh.G = static_cast<uint32_t>(sms);
+    sh.per = static_cast<uint32_t>((N + sh.G - 1) / sh.G);
+    sh.pad = 0;
+    // one member per thread in the common case: room for a quarter more than the mean run
+    const uint32_t want = (K + sh.G - 1) / sh.G;
+    uint32_t thr = ((want + want / 4u + 31u) / 32u) * 32u;
+    if (thr < 32u) thr = 32u;
+    if (thr > 512u) thr = 512u;
+    const size_t base = 2 * static_cast<size_t>(tab_stride) + 2ull * thr * P;
+    const size_t res_bytes = base + static_cast<size_t>(sh.per) * SB;
+    const size_t x_bytes = base + static_cast<size_t>(thr) * SB + ((static_cast<size_t>(sh.per) + 15u) & ~size_t(15));
+    sh.res = res_bytes + 2048 <= static_cast<size_t>(max_optin) ? 1u : 0u;
+    const size_t bytes = sh.res ? res_bytes : x_bytes;
+    if (bytes + 2048 > static_cast<size_t>(max_optin)) return false;
+    const void *fn = owned_fn(SB, P, sh.res != 0);
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes)) !=
+        cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, static_cast<int>(thr), bytes) != cudaSuccess ||
+        per_sm < 1)
+        return false;
+    *grid = static_cast<int>(sh.G);
+    *threads = thr;
+    *smem = bytes;
+    *static_cast<OwnedShape *>(shape_out) = sh;
+    return true;
+}
+
+cudaError_t launch_route(const StepArgs &a, const void *shape, uint32_t *perm_m, uint32_t *perm_s, uint32_t *perm_o,
+                         uint32_t *off, cudaStream_t s) {
+    const OwnedShape &sh = *static_cast<const OwnedShape *>(shape);
+    const size_t smem = (sh.G + 1) * sizeof(uint32_t);
+    k_route<<<a.n_sets, 1024, smem, s>>>(a.idx, a.outcome, a.n_sets, a.K, a.n_sessions, sh.G, sh.per, perm_m,
+                                          perm_s, perm_o, off, a.dev);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_chain_owned(const StepArgs &a, int SB, int P, int grid, uint32_t threads, size_t smem,
+                               const void *shape, const uint32_t *perm_m, const uint32_t *perm_s,
+                               const uint32_t *perm_o, const uint32_t *off, cudaStream_t s) {
+    const OwnedShape &sh = *static_cast<const OwnedShape *>(shape);
+    StepArgs aa = a;
+    OwnedShape shc = sh;
+    void *args[] = {&aa, &shc, &perm_m, &perm_s, &perm_o, &off};
+    return cudaLaunchCooperativeKernel(owned_fn(SB, P, sh.res != 0), dim3(grid), dim3(threads), args, smem, s);
 }
 
 cudaError_t launch_empty_cohorts(const StepArgs &a, cudaStream_t s) {

@@ -173,7 +173,7 @@ def test_launch_floor_probes_run(g, rc):
         rc.rc_free(ctx)
 
 
-@pytest.mark.parametrize("kernel", ["split", "tma", "plain"])
+@pytest.mark.parametrize("kernel", ["owned", "split", "tma", "plain"])
 @pytest.mark.parametrize("SB,P", [(16, 32), (16, 64), (64, 128), (64, 32)])
 @pytest.mark.parametrize("K,N,identity", [(1032, 5000, False), (4104, 9001, False), (4104, 4200, False),
                                           (2048, 2048, True), (65536, 70000, False), (65536, 1 << 20, False)])
@@ -181,6 +181,7 @@ def test_persistent_grid_kernels(g, rc, monkeypatch, kernel, SB, P, K, N, identi
     """The cooperative persistent kernels: split-phase (explicit sessions, K a
     multiple of 8), TMA-fed and plain, on member counts that do not split
     evenly over SMs, with sessions recurring from step to step (N near K)."""
+    monkeypatch.setenv("RC_OWNED", "1" if kernel == "owned" else "0")
     monkeypatch.setenv("RC_SPLIT", "1" if kernel == "split" else "0")
     monkeypatch.setenv("RC_NO_TMA", "1" if kernel == "plain" else "0")
     S = 256 if SB == 64 else 64
@@ -191,12 +192,12 @@ def test_persistent_grid_kernels(g, rc, monkeypatch, kernel, SB, P, K, N, identi
     g.assert_same(got, want, f"grid {kernel} K={K} N={N} SB={SB} P={P}")
 
 
-@pytest.mark.parametrize("tma", [True, False])
-@pytest.mark.parametrize("split", [True, False])
-def test_grid_barrier_wait_is_bounded_both_kernels(g, rc, monkeypatch, tma, split):
+@pytest.mark.parametrize("kernel", ["owned", "split", "tma", "plain"])
+def test_grid_barrier_wait_is_bounded_every_grid_kernel(g, rc, monkeypatch, kernel):
     import torch
-    monkeypatch.setenv("RC_NO_TMA", "0" if tma else "1")
-    monkeypatch.setenv("RC_SPLIT", "1" if split else "0")
+    monkeypatch.setenv("RC_OWNED", "1" if kernel == "owned" else "0")
+    monkeypatch.setenv("RC_SPLIT", "1" if kernel == "split" else "0")
+    monkeypatch.setenv("RC_NO_TMA", "1" if kernel == "plain" else "0")
     K, S, SB, P, n = 8192, 16, 16, 64, 4
     tables, state0, outc, pay, idx = _inputs(19, K, S, SB, P, 2, N=9000)
     ctx = rc.rc_init(S, tables, SB, P, K, 9000, torch.cuda.current_stream())
@@ -219,20 +220,20 @@ def test_grid_barrier_wait_is_bounded_both_kernels(g, rc, monkeypatch, tma, spli
         rc.rc_free(ctx)
 
 
-@pytest.mark.parametrize("split", [True, False])
+@pytest.mark.parametrize("kernel", ["owned", "split", "plain"])
 @pytest.mark.parametrize("P", [32, 64, 128])
 @pytest.mark.parametrize("K,N", [(8, 9), (64, 67), (64, 128), (256, 259), (256, 512), (496, 1000), (512, 513),
-                                 (100, 300)])
-def test_single_cta_repeated_sessions(g, rc, monkeypatch, split, P, K, N):
-    """Sessions that recur in consecutive steps at other member positions: the
-    split-phase chain must finish them after the step that wrote them, not
-    from records read early."""
-    monkeypatch.setenv("RC_SPLIT", "1" if split else "0")
+                                 (100, 300), (256, 1 << 20)])
+def test_small_cohort_repeated_sessions(g, rc, monkeypatch, kernel, P, K, N):
+    """Sessions that recur in consecutive steps at other member positions: each
+    persistent kernel must see the records the previous step wrote."""
+    monkeypatch.setenv("RC_OWNED", "1" if kernel == "owned" else "0")
+    monkeypatch.setenv("RC_SPLIT", "1" if kernel == "split" else "0")
     tables, state0, outc, pay, idx = _inputs(60 + K % 13 + P, K, 64, 16, P, 40, N=N)
     n = 40
     want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=1)
     got = g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K, sel0=1)
-    g.assert_same(got, want, f"split={split} K={K} N={N} P={P}")
+    g.assert_same(got, want, f"{kernel} K={K} N={N} P={P}")
 
 
 @pytest.mark.parametrize("pipe", [True, False])
