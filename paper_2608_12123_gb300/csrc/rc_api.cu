@@ -89,9 +89,12 @@ struct rc_ctx {
     uint32_t last_launches = 0;
     bool no_tma = false;   // RC_NO_TMA=1 in the environment selects the plain grid kernel
     bool no_pipe = false;   // RC_NO_PIPE=1 selects the plain single-CTA kernel
+    bool no_link = false;   // RC_NO_LINK=1 turns off the linked single-CTA kernels
+    bool no_prod = false;   // RC_NO_PROD=1 keeps the linked kernel without a producer warp
     bool use_split = false;  // RC_SPLIT=1 selects the split-phase chain (slower on GB300 so far)
     bool use_owned = false;  // RC_OWNED=1 selects the session-owned chain
     Buf route_buf;           // session-owned chain: routed member lists
+    Buf link_buf;            // linked single-CTA chain: n_sets * K link words
     Buf marks;              // split-phase cohort marks (3 * n_sessions words)
     long long *trace = nullptr;
     uint64_t trace_entries = 0;
@@ -390,6 +393,7 @@ int run_persist(rc_ctx *c, const rc::StepArgs &a) {
             uint32_t *ps = pm + nev, *po = ps + nev, *off = po + nev;
             RC_CUDA(c, cudaMemsetAsync(c->dev->slot4, 0, sizeof(c->dev->slot4), c->stream));
             RC_CUDA(c, cudaMemsetAsync(&c->dev->abort, 0, sizeof(uint32_t), c->stream));
+            c->last_launches = 2;  // routing pass + chain
             RC_CUDA(c, rc::launch_route(a, shape, pm, ps, po, off, c->stream));
             RC_CUDA(c, rc::launch_chain_owned(a, c->SB, c->P, grid, threads, smem, shape, pm, ps, po, off,
                                               c->stream));
@@ -412,6 +416,19 @@ int run_persist(rc_ctx *c, const rc::StepArgs &a) {
             RC_CUDA(c, rc::launch_chain_split(a, c->SB, c->P, grid, threads, smem, shape,
                                               static_cast<uint32_t *>(c->marks.p), c->stream));
             RC_CUDA(c, cudaMemsetAsync(&c->dev->skip_arrival, 0, sizeof(uint32_t), c->stream));
+            return RC_OK;
+        }
+    }
+    if (a.idx && !c->no_pipe && !c->no_link) {
+        size_t smem = 0;
+        alignas(8) unsigned char shape[16];
+        if (rc::chain_cta_link_plan(c->SB, c->P, a.K, c->n_sessions, c->tab_stride, !c->no_prod, &smem, shape)) {
+            int rc = ensure(c, c->link_buf, static_cast<size_t>(a.n_sets) * a.K * sizeof(uint32_t));
+            if (rc != RC_OK) return rc;
+            uint32_t *lnk = static_cast<uint32_t *>(c->link_buf.p);
+            c->last_launches = 2;  // link pass + chain
+            RC_CUDA(c, rc::launch_link(a, lnk, c->stream));
+            RC_CUDA(c, rc::launch_chain_cta_link(a, c->SB, c->P, smem, shape, lnk, c->stream));
             return RC_OK;
         }
     }
@@ -556,6 +573,10 @@ int rc_init(rc_ctx **out, uint32_t S, const uint8_t *table, uint32_t state_bytes
         c->no_tma = v && v[0] == '1';
         const char *w = std::getenv("RC_NO_PIPE");
         c->no_pipe = w && w[0] == '1';
+        const char *z = std::getenv("RC_NO_LINK");
+        c->no_link = z && z[0] == '1';
+        const char *q = std::getenv("RC_NO_PROD");
+        c->no_prod = q && q[0] == '1';
         const char *x = std::getenv("RC_SPLIT");
         c->use_split = x && x[0] == '1';
         const char *y = std::getenv("RC_OWNED");
@@ -634,7 +655,8 @@ int rc_chain(rc_ctx *c, uint32_t n_steps, rc_mechanism mech, void *state, const 
         c->last_launches = floor ? 0u : 1u;
     } else {
         // kernel executions: one per step, two per step for the nested control
-        // (launcher + child), one for the persistent kernel
+        // (launcher + child), one for the persistent kernel (two where it
+        // starts with a pass over the event ring)
         c->last_launches = mech == RC_MECH_RESIDENT_PERSIST ? 1u
                            : mech == RC_MECH_FIXED_NESTED  ? 2u * n_steps
                                                            : n_steps;
@@ -663,7 +685,7 @@ int rc_free(rc_ctx *c) {
     c->cond.reset();
     c->floor.reset();
     c->nested.reset();
-    for (Buf *b : {&c->st_outcome, &c->st_payload, &c->st_idx, &c->st_dec, &c->st_eff, &c->st_log, &c->marks, &c->route_buf})
+    for (Buf *b : {&c->st_outcome, &c->st_payload, &c->st_idx, &c->st_dec, &c->st_eff, &c->st_log, &c->marks, &c->route_buf, &c->link_buf})
         if (b->p) cudaFree(b->p);
     if (c->d_tables) cudaFree(c->d_tables);
     if (c->dev) cudaFree(c->dev);

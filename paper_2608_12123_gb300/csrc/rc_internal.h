@@ -79,11 +79,20 @@ cudaError_t launch_step(const StepArgs &a, int state_bytes, int payload_bytes, i
 // Persistent chains.  The single-CTA form takes K <= 512; the grid form is a
 // cooperative launch of `grid` CTAs.
 cudaError_t launch_chain_cta(const StepArgs &a, int state_bytes, int payload_bytes, cudaStream_t s);
-// Pipelined single-CTA chains (identity sessions: records in registers;
-// explicit indices, 16-byte records, K <= 512: D-step prefetch with a shared
-// write-back table).  *launched is false when neither applies.
+// Pipelined single-CTA chain for identity sessions (records in registers).
+// *launched is false when it does not apply.
 cudaError_t launch_chain_cta_fast(const StepArgs &a, int state_bytes, int payload_bytes, cudaStream_t s,
                                   bool *launched);
+// Single-CTA chains with explicit indices and the record gather ahead of its
+// step (K <= 512): launch_link fills lnk (n_sets * K words) with each
+// member's position in the two previous cohorts, then the chain runs (the
+// producer-warp form when allow_prod and K is a multiple of 8 and it fits).
+// shape_out points to 16 bytes of opaque shape.
+bool chain_cta_link_plan(int state_bytes, int payload_bytes, uint32_t K, uint64_t n_sessions, uint32_t tab_stride,
+                         bool allow_prod, size_t *smem, void *shape_out);
+cudaError_t launch_link(const StepArgs &a, uint32_t *lnk, cudaStream_t s);
+cudaError_t launch_chain_cta_link(const StepArgs &a, int state_bytes, int payload_bytes, size_t smem,
+                                  const void *shape, const uint32_t *lnk, cudaStream_t s);
 cudaError_t chain_grid_size(int state_bytes, int payload_bytes, uint32_t K, int *grid);
 cudaError_t launch_chain_grid(const StepArgs &a, int state_bytes, int payload_bytes, int grid,
                               cudaStream_t s);

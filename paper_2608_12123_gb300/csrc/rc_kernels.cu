@@ -153,6 +153,30 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
     return done != 0u;
 }
 
+// Spin-wait clock: the first call stamps t0, later calls report whether
+// limit_ns has passed since then (the clock is not read on the fast path).
+__device__ __forceinline__ bool timed_out(uint64_t &t0, uint64_t limit_ns) {
+    const uint64_t now = globaltimer_ns();
+    if (t0 == 0) {
+        t0 = now;
+        return false;
+    }
+    return now - t0 > limit_ns;
+}
+
+// Bounded wait for an mbarrier phase.  The clock is read only once the phase
+// is found incomplete, so a phase that has already completed costs one
+// try_wait.  False when limit_ns ran out.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity, uint64_t limit_ns) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = globaltimer_ns();
+    uint32_t spins = 0;
+    while (!mbar_try_wait(bar, parity)) {
+        if ((++spins & 255u) == 0u && globaltimer_ns() - t0 > limit_ns) return false;
+    }
+    return true;
+}
+
 // L2 eviction-priority policies (applied to whole accesses).
 __device__ __forceinline__ uint64_t policy_evict_first() {
     uint64_t p;
@@ -563,7 +587,7 @@ __global__ void __launch_bounds__(kGridThreads) k_chain_grid(StepArgs a) {
             __threadfence();
             const bool skip = (n == 0 && blockIdx.x == 1 && ld_volatile_u32(&a.dev->skip_arrival) != 0u);
             if (!skip) red_release_add_u64(word, (1ull << 32) | c);
-            const uint64_t t0 = globaltimer_ns();
+            uint64_t t0 = 0;
             unsigned long long w;
             uint32_t spins = 0;
             for (;;) {
@@ -574,7 +598,7 @@ __global__ void __launch_bounds__(kGridThreads) k_chain_grid(StepArgs a) {
                         s_abort = 1;
                         break;
                     }
-                    if (globaltimer_ns() - t0 > limit) {
+                    if (timed_out(t0, limit)) {
                         latch_error(a.dev, DEV_E_TIMEOUT, n, blockIdx.x);
                         atomicExch(&a.dev->abort, 1u);
                         s_abort = 1;
@@ -678,14 +702,7 @@ __global__ void __launch_bounds__(512, 1)
         s_pend_step[st] = j;
     };
     // bounded wait for stage st's copies; false when it gave up
-    auto wait_stage = [&](uint32_t st, uint32_t parity) -> bool {
-        const uint64_t t0 = globaltimer_ns();
-        uint32_t spins = 0;
-        while (!mbar_try_wait(&bar[st], parity)) {
-            if ((++spins & 255u) == 0u && globaltimer_ns() - t0 > limit) return false;
-        }
-        return true;
-    };
+    auto wait_stage = [&](uint32_t st, uint32_t parity) -> bool { return mbar_wait_bounded(&bar[st], parity, limit); };
 
     if (tid == 0) {
         mbar_init(&bar[0], 1);
@@ -746,7 +763,7 @@ __global__ void __launch_bounds__(512, 1)
                 }
             }
             if (trace) trace[n * 8 + 4] = clock64();
-            const uint64_t t0 = globaltimer_ns();
+            uint64_t t0 = 0;
             unsigned long long w;
             uint32_t spins = 0;
             for (;;) {
@@ -757,7 +774,7 @@ __global__ void __launch_bounds__(512, 1)
                         s_abort = 1;
                         break;
                     }
-                    if (globaltimer_ns() - t0 > limit) {
+                    if (timed_out(t0, limit)) {
                         latch_error(a.dev, DEV_E_TIMEOUT, n, blockIdx.x);
                         atomicExch(&a.dev->abort, 1u);
                         s_abort = 1;
@@ -801,6 +818,468 @@ __global__ void __launch_bounds__(512, 1)
     if (blockIdx.x == 0 && tid == 0) {
         if (a.n_steps > 0) a.dev->sel = sel;
         a.dev->step = a.n_steps;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Links between consecutive cohorts of the event ring (explicit session
+// indices, K <= 512).  For member m of cohort j, lnk[j][m] holds 1 + the
+// position of the same session in cohort j - 1 (low 16 bits) and in cohort
+// j - 2 (high 16 bits), 0 where it is absent; cohorts are taken modulo n_sets,
+// as the chain takes them.  Sessions are distinct within a cohort, so each
+// position is unique; an index >= N is never linked (its member is rejected
+// anyway).  One CTA per cohort at a time, two open-addressing tables in shared
+// memory (1024 slots for at most 512 keys, so every probe sequence ends).
+// ---------------------------------------------------------------------------
+constexpr uint32_t kLinkSlots = 1024;
+constexpr uint32_t kLinkEmpty = 0xFFFFFFFFu;
+
+__device__ __forceinline__ uint32_t link_hash(uint32_t s) { return (s * 0x9E3779B1u) >> 22; }
+
+__global__ void __launch_bounds__(512) k_link(const uint32_t *idx, uint32_t n_sets, uint32_t K, uint64_t N,
+                                              uint32_t *lnk) {
+    __shared__ uint32_t key[2][kLinkSlots];
+    __shared__ uint16_t pos[2][kLinkSlots];
+    for (uint32_t j = blockIdx.x; j < n_sets; j += gridDim.x) {
+        for (uint32_t i = threadIdx.x; i < 2 * kLinkSlots; i += blockDim.x) (&key[0][0])[i] = kLinkEmpty;
+        __syncthreads();
+        for (uint32_t t = 0; t < 2; ++t) {
+            const uint32_t src = static_cast<uint32_t>((static_cast<uint64_t>(j) + 2ull * n_sets - 1u - t) % n_sets);
+            for (uint32_t m = threadIdx.x; m < K; m += blockDim.x) {
+                const uint32_t s = __ldg(idx + static_cast<size_t>(src) * K + m);
+                if (s >= N) continue;
+                uint32_t h = link_hash(s);
+                for (uint32_t probe = 0; probe < kLinkSlots; ++probe) {
+                    const uint32_t prev = atomicCAS(&key[t][h], kLinkEmpty, s);
+                    if (prev == kLinkEmpty || prev == s) {
+                        pos[t][h] = static_cast<uint16_t>(m);
+                        break;
+                    }
+                    h = (h + 1u) & (kLinkSlots - 1u);
+                }
+            }
+        }
+        __syncthreads();
+        for (uint32_t m = threadIdx.x; m < K; m += blockDim.x) {
+            const uint32_t s = __ldg(idx + static_cast<size_t>(j) * K + m);
+            uint32_t l = 0;
+            if (s < N) {
+#pragma unroll
+                for (uint32_t t = 0; t < 2; ++t) {
+                    uint32_t h = link_hash(s);
+                    for (uint32_t probe = 0; probe < kLinkSlots; ++probe) {
+                        const uint32_t k = key[t][h];
+                        if (k == s) {
+                            l |= (static_cast<uint32_t>(pos[t][h]) + 1u) << (16u * t);
+                            break;
+                        }
+                        if (k == kLinkEmpty) break;
+                        h = (h + 1u) & (kLinkSlots - 1u);
+                    }
+                }
+            }
+            lnk[static_cast<size_t>(j) * K + m] = l;
+        }
+        __syncthreads();
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Persistent chain, one CTA, explicit session indices (K <= 512), with the
+// state gather off the critical path.  The record of a step-n member is
+// fetched (per-thread asynchronous copy) at the top of step n - 2, when every
+// store of steps <= n - 3 is visible to the CTA.  A member whose session was
+// also in step n - 1 or n - 2 (its link) takes that step's result from the
+// shared record ring instead: each step leaves there, in its own slot, the
+// record it wrote, or the record as it stood for a rejected member.
+//
+// Every copy is a per-thread asynchronous copy of the thread's own member:
+// records, outcomes and payload rows two steps ahead, session indices and
+// links four.  The decision is the block barrier's own count (bar.red.popc),
+// the only block barrier of a step.  This form takes any K <= 512; for K a
+// multiple of 8, k_chain_cta_prod below moves every copy to a producer warp.
+// ---------------------------------------------------------------------------
+constexpr uint32_t kLinkRI = 5;  // index / link slots
+constexpr uint32_t kLinkRP = 3;  // outcome / payload slots
+constexpr uint32_t kLinkRR = 5;  // record slots
+
+struct LinkShape {
+    uint32_t box_rows;   // payload rows per tensor tile (producer form)
+    uint32_t n_boxes;    // tiles per step (producer form)
+    uint32_t stage_pay;  // payload bytes per slot (a multiple of 1024)
+    uint32_t prod;       // 1: k_chain_cta_prod, 0: k_chain_cta_link
+};
+
+template <int SB, int P>
+__global__ void __launch_bounds__(512, 1) k_chain_cta_link(StepArgs a, const uint32_t *lnk, LinkShape sh) {
+    constexpr uint32_t NC = P / 16;
+    constexpr int NV = SB / 16;
+    constexpr uint32_t RI = kLinkRI, RP = kLinkRP, RR = kLinkRR;
+    extern __shared__ uint8_t dsm_raw[];
+    const uint32_t raw = smem_addr(dsm_raw);
+    uint8_t *const base = dsm_raw + (((raw + 1023u) & ~1023u) - raw);
+    const uint32_t K = a.K;
+    const uint32_t Kp = (K + 3u) & ~3u;
+    const uint32_t tid = threadIdx.x;
+    const uint32_t nst = a.n_steps;
+    // layout: [payload slots][records][indices][links][outcomes][tables]
+    uint8_t *const pay = base;
+    uint4 *const rec = reinterpret_cast<uint4 *>(base + static_cast<size_t>(RP) * sh.stage_pay);  // [RR][Kp][NV]
+    uint32_t *const sidx = reinterpret_cast<uint32_t *>(rec + static_cast<size_t>(RR) * Kp * NV);  // [RI][Kp]
+    uint32_t *const slnk = sidx + RI * Kp;                                                         // [RI][Kp]
+    uint32_t *const sout = slnk + RI * Kp;                                                         // [RP][Kp]
+    uint8_t *const tab = reinterpret_cast<uint8_t *>(sout + RP * Kp);
+    const bool act = tid < K;
+    const uint32_t m = tid;
+    long long *trace = (a.trace && tid == 0) ? a.trace : nullptr;
+
+    auto issue_idx = [&](uint32_t j) {  // session index and link of step j
+        if (!act || j >= nst) return;
+        const size_t e = static_cast<size_t>(j % a.n_sets) * K + m;
+        cp_async4(&sidx[(j % RI) * Kp + m], a.idx + e);
+        cp_async4(&slnk[(j % RI) * Kp + m], lnk + e);
+    };
+    auto issue_rec = [&](uint32_t j) {  // record (by the index already here) and outcome of step j
+        if (!act || j >= nst) return;
+        const size_t e = static_cast<size_t>(j % a.n_sets) * K + m;
+        const uint32_t s = sidx[(j % RI) * Kp + m];
+        if (s < a.n_sessions) {
+            const uint4 *rp = reinterpret_cast<const uint4 *>(a.state + static_cast<size_t>(s) * SB);
+            uint4 *dst = rec + (static_cast<size_t>(j % RR) * Kp + m) * NV;
+#pragma unroll
+            for (int k = 0; k < NV; ++k) cp_async16(dst + k, rp + k);
+        }
+        cp_async4(&sout[(j % RP) * Kp + m], a.outcome + e);
+        const uint4 *src = reinterpret_cast<const uint4 *>(a.payload + e * P);
+        uint4 *ring = reinterpret_cast<uint4 *>(pay + static_cast<size_t>(j % RP) * sh.stage_pay);
+#pragma unroll
+        for (uint32_t k = 0; k < NC; ++k) cp_async16(ring + pay_chunk<P>(m, k), src + k);
+    };
+    stage_tables(tab, a.tables, a.tab_stride, 2, 0);
+    uint32_t sel = ld_volatile_u32(&a.dev->sel) & 1u;
+    // prologue: indices of steps 0..3, then the records of steps 0 and 1 in
+    // the group pattern of the loop (record group, index group) per step
+    for (uint32_t j = 0; j < 4; ++j) issue_idx(j);
+    cp_async_commit();
+    cp_async_wait<0>();
+    issue_rec(0);
+    cp_async_commit();
+    cp_async_commit();
+    issue_rec(1);
+    cp_async_commit();
+    cp_async_commit();
+    __syncthreads();
+
+    for (uint32_t n = 0; n < nst; ++n) {
+        if (trace) trace[n * 8 + 0] = clock64();
+        cp_async_wait<2>();  // record, outcome and payload of step n; index of step n + 2
+        if (trace) trace[n * 8 + 1] = clock64();
+        issue_rec(n + 2u);
+        cp_async_commit();
+        issue_idx(n + 4u);
+        cp_async_commit();
+        if (trace) trace[n * 8 + 2] = clock64();
+        uint32_t odd = 0;
+        if (act) {
+            const uint32_t s = sidx[(n % RI) * Kp + m];
+            const uint32_t l = slnk[(n % RI) * Kp + m];
+            const uint32_t o = sout[(n % RP) * Kp + m];
+            uint4 *mine = rec + (static_cast<size_t>(n % RR) * Kp + m) * NV;
+            if (s >= a.n_sessions) {
+                latch_error(a.dev, DEV_E_INDEX, n, m);
+            } else {
+                const uint32_t p1 = l & 0xFFFFu, p2 = l >> 16;
+                const uint4 *src = mine;
+                if (p1 != 0u && n >= 1u)
+                    src = rec + (static_cast<size_t>((n - 1u) % RR) * Kp + (p1 - 1u)) * NV;
+                else if (p2 != 0u && n >= 2u)
+                    src = rec + (static_cast<size_t>((n - 2u) % RR) * Kp + (p2 - 1u)) * NV;
+                uint4 r[NV];
+#pragma unroll
+                for (int k = 0; k < NV; ++k) r[k] = src[k];
+                const uint32_t x = r[0].x;
+                if (x >= a.S || o >= 8u) {
+                    latch_error(a.dev, DEV_E_STATE, n, m);
+                    if (src != mine) {
+#pragma unroll
+                        for (int k = 0; k < NV; ++k) mine[k] = r[k];
+                    }
+                } else {
+                    uint4 pw[NC];
+                    const uint4 *ring = reinterpret_cast<const uint4 *>(pay + static_cast<size_t>(n % RP) * sh.stage_pay);
+#pragma unroll
+                    for (uint32_t k = 0; k < NC; ++k) pw[k] = ring[pay_chunk<P>(m, k)];
+                    const uint64_t rk = route_key<P>(x, o, pw);
+                    const uint32_t y = tab[sel * a.tab_stride + x * 8u + o];
+                    r[0].x = y;
+                    r[0].y = r[0].y + 1u;
+                    mix_acc<SB>(r, rk);
+                    uint4 *rp = reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(s) * SB);
+#pragma unroll
+                    for (int k = 0; k < NV; ++k) {
+                        mine[k] = r[k];
+                        rp[k] = r[k];
+                    }
+                    const size_t slot = static_cast<size_t>(n) * K + m;
+                    if (a.effects) {
+                        uint4 e;
+                        e.x = static_cast<uint32_t>(rk);
+                        e.y = static_cast<uint32_t>(rk >> 32);
+                        e.z = s;
+                        e.w = y | (o << 16) | (sel << 24);
+                        __stcs(reinterpret_cast<uint4 *>(a.effects) + slot, e);
+                    }
+                    if (a.state_log) {
+                        uint4 *lp = reinterpret_cast<uint4 *>(a.state_log + slot * SB);
+#pragma unroll
+                        for (int k = 0; k < NV; ++k) __stcs(lp + k, r[k]);
+                    }
+                    odd = static_cast<uint32_t>(rk & 1u);
+                }
+            }
+        }
+        if (trace) trace[n * 8 + 3] = clock64();
+        // the block barrier counts the odd keys; it also publishes this step's
+        // record slots and orders its state stores
+        const uint32_t total = static_cast<uint32_t>(__syncthreads_count(odd));
+        if (trace) trace[n * 8 + 4] = clock64();
+        sel = total > K / 2u ? 1u : 0u;
+        if (tid == 0 && a.decisions) a.decisions[n] = sel;
+    }
+    cp_async_wait<0>();
+    if (tid == 0) {
+        if (nst > 0) a.dev->sel = sel;
+        a.dev->step = nst;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Persistent chain, one CTA, explicit session indices, K a multiple of 8 up
+// to 512, with a producer warp for the streams.  Warps 0 .. ceil(K/32) - 1
+// transition one member per thread; lane 0 of the last warp, in region n
+// (from the block barrier of step n - 1 to that of step n):
+//   - stores decision n - 1;
+//   - issues the outcome, session-index and link runs of step n + 5 (1-D bulk
+//     copies onto mbarrier W[(n + 5) % 6]) and the payload tiles of step
+//     n + 3 (tensor copies onto mbarrier P[(n + 3) % 4]);
+//   - waits (bounded) for the runs of step n + 3 and the tiles of step n + 1.
+// The barrier of step n then tells every member warp that what it reads in
+// region n + 1 has landed, so member warps never wait on an mbarrier and
+// never issue a load for the streams.
+//
+// The one scattered access, the gather of state records, stays with the
+// member warps: in step n each thread gathers (asynchronous copy) the record
+// of its member of step n + 2, even warps before their transition and odd
+// warps after it.  The gather of step j thus starts once every store of
+// steps <= j - 3 is visible; a member whose session was in step j - 1 or
+// j - 2 takes that step's result from the shared record ring (links from
+// k_link), as in k_chain_cta_link.  The decision is the barrier's own count.
+// A producer wait that runs out latches RC_E_TIMEOUT; the CTA stops after
+// that step, the producer first waiting (bounded) for the copies it still
+// has in flight.
+// ---------------------------------------------------------------------------
+constexpr uint32_t kProdRW = 6;  // word slots (issued five steps ahead)
+constexpr uint32_t kProdRP = 4;  // payload slots (issued three steps ahead)
+constexpr uint32_t kProdRR = 5;  // record slots (two ahead, two of forwarding)
+
+template <int SB, int P>
+__global__ void __launch_bounds__(544, 1)
+    k_chain_cta_prod(const __grid_constant__ CUtensorMap tmap, StepArgs a, const uint32_t *lnk, LinkShape sh) {
+    constexpr int NV = SB / 16;
+    constexpr uint32_t RW = kProdRW, RP = kProdRP, RR = kProdRR;
+    extern __shared__ uint8_t dsm_raw[];
+    __shared__ __align__(8) uint64_t wbar[RW];
+    __shared__ __align__(8) uint64_t pbar[RP];
+    __shared__ uint32_t s_ab[2];
+    const uint32_t raw = smem_addr(dsm_raw);
+    uint8_t *const base = dsm_raw + (((raw + 1023u) & ~1023u) - raw);
+    const uint32_t K = a.K;
+    const uint32_t Kw = (K + 31u) & ~31u;  // member threads; the producer warp follows
+    const uint32_t tid = threadIdx.x;
+    const bool prod = tid >= Kw;
+    const bool early = ((tid >> 5) & 1u) == 0u;  // even member warps gather before their transition
+    const uint32_t nst = a.n_steps;
+    const uint64_t limit = a.dev->wait_ns;
+    // layout: [payload slots][records][word slots: outcome, index, link][tables]
+    uint8_t *const pay = base;
+    uint4 *const rec = reinterpret_cast<uint4 *>(base + static_cast<size_t>(RP) * sh.stage_pay);  // [RR][K][NV]
+    uint32_t *const words = reinterpret_cast<uint32_t *>(rec + static_cast<size_t>(RR) * K * NV);  // [RW][3][K]
+    uint8_t *const tab = reinterpret_cast<uint8_t *>(words + static_cast<size_t>(RW) * 3 * K);
+    auto word_of = [&](uint32_t j, uint32_t which) { return words + (static_cast<size_t>(j % RW) * 3 + which) * K; };
+    const uint64_t stream_pol = policy_evict_first();
+    long long *trace = (a.trace && tid == 0) ? a.trace : nullptr;
+
+    // producer lane 0 only
+    auto issue_words = [&](uint32_t j) {
+        if (j >= nst) return;
+        const size_t e0 = static_cast<size_t>(j % a.n_sets) * K;
+        uint64_t *b = &wbar[j % RW];
+        mbar_arrive_expect_tx(b, 3u * K * 4u);
+        bulk_load_hint(word_of(j, 0), a.outcome + e0, K * 4u, b, stream_pol);
+        bulk_load_hint(word_of(j, 1), a.idx + e0, K * 4u, b, stream_pol);
+        bulk_load_hint(word_of(j, 2), lnk + e0, K * 4u, b, stream_pol);
+    };
+    auto issue_pay = [&](uint32_t j) {
+        if (j >= nst) return;
+        const uint32_t st = j % RP;
+        const int32_t row0 = static_cast<int32_t>((j % a.n_sets) * K);
+        mbar_arrive_expect_tx(&pbar[st], sh.n_boxes * sh.box_rows * P);
+        for (uint32_t b = 0; b < sh.n_boxes; ++b)
+            tma_load_2d_hint(pay + static_cast<size_t>(st) * sh.stage_pay + b * sh.box_rows * P, &tmap, 0,
+                             row0 + static_cast<int32_t>(b * sh.box_rows), &pbar[st], stream_pol);
+    };
+    auto landed_words = [&](uint32_t j) { return j >= nst || mbar_wait_bounded(&wbar[j % RW], (j / RW) & 1u, limit); };
+    auto landed_pay = [&](uint32_t j) { return j >= nst || mbar_wait_bounded(&pbar[j % RP], (j / RP) & 1u, limit); };
+    // member thread: gather its record of step j (one commit group, empty past the end);
+    // the index run of step j is known to have landed
+    auto gather = [&](uint32_t j) {
+        if (j < nst && tid < K) {
+            const uint32_t s = word_of(j, 1)[tid];
+            if (s < a.n_sessions) {
+                const uint4 *rp = reinterpret_cast<const uint4 *>(a.state + static_cast<size_t>(s) * SB);
+                uint4 *dst = rec + (static_cast<size_t>(j % RR) * K + tid) * NV;
+#pragma unroll
+                for (int k = 0; k < NV; ++k) cp_async16(dst + k, rp + k);
+            }
+        }
+        cp_async_commit();
+    };
+
+    if (tid == 0) {
+        for (uint32_t i = 0; i < RW; ++i) mbar_init(&wbar[i], 1);
+        for (uint32_t i = 0; i < RP; ++i) mbar_init(&pbar[i], 1);
+        fence_mbar_init();
+        s_ab[0] = 0;
+        s_ab[1] = 0;
+    }
+    stage_tables(tab, a.tables, a.tab_stride, 2, 0);
+    uint32_t sel = ld_volatile_u32(&a.dev->sel) & 1u;
+    __syncthreads();
+    // prologue: runs of steps 0..4 and tiles of steps 0..2 go out; the runs
+    // of steps 0..2 and the tiles of step 0 are waited for; the member warps
+    // then gather the records of steps 0 and 1
+    if (tid == Kw) {
+        for (uint32_t j = 0; j + 1u < RW; ++j) issue_words(j);
+        for (uint32_t j = 0; j + 1u < RP; ++j) issue_pay(j);
+        if (!(landed_words(0) && landed_words(1) && landed_words(2) && landed_pay(0))) {
+            latch_error(a.dev, DEV_E_TIMEOUT, 0, tid);
+            s_ab[0] = 1;
+        }
+    }
+    __syncthreads();
+    const bool started = s_ab[0] == 0u;  // false: the prologue gave up a wait, no step runs
+    if (started && !prod) {
+        gather(0);
+        gather(1);
+    }
+
+    // A thread that gives up a wait in region n raises s_ab[n & 1]; all
+    // threads read it after the barrier of step n, before anyone can write it
+    // again.
+    uint32_t n = 0;
+    for (; started && n < nst; ++n) {
+        uint32_t odd = 0;
+        if (prod) {
+            if (tid == Kw) {
+                if (n > 0 && a.decisions) a.decisions[n - 1u] = sel;
+                issue_words(n + RW - 1u);
+                issue_pay(n + RP - 1u);
+                if (!(landed_words(n + 3u) && landed_pay(n + 1u))) {
+                    latch_error(a.dev, DEV_E_TIMEOUT, n, tid);
+                    s_ab[n & 1u] = 1;
+                }
+            }
+        } else {
+            if (trace) trace[n * 8 + 0] = clock64();
+            if (early) {
+                gather(n + 2u);
+                cp_async_wait<2>();  // this thread's record of step n
+            } else {
+                cp_async_wait<1>();
+            }
+            if (trace) trace[n * 8 + 1] = clock64();
+            if (tid < K) {
+                const uint32_t m = tid;
+                const uint32_t o = word_of(n, 0)[m];
+                const uint32_t s = word_of(n, 1)[m];
+                const uint32_t l = word_of(n, 2)[m];
+                uint4 *mine = rec + (static_cast<size_t>(n % RR) * K + m) * NV;
+                if (s >= a.n_sessions) {
+                    latch_error(a.dev, DEV_E_INDEX, n, m);
+                } else {
+                    const uint32_t p1 = l & 0xFFFFu, p2 = l >> 16;
+                    const uint4 *src = mine;
+                    if (p1 != 0u && n >= 1u)
+                        src = rec + (static_cast<size_t>((n - 1u) % RR) * K + (p1 - 1u)) * NV;
+                    else if (p2 != 0u && n >= 2u)
+                        src = rec + (static_cast<size_t>((n - 2u) % RR) * K + (p2 - 1u)) * NV;
+                    uint4 r[NV];
+#pragma unroll
+                    for (int k = 0; k < NV; ++k) r[k] = src[k];
+                    const uint32_t x = r[0].x;
+                    if (x >= a.S || o >= 8u) {
+                        latch_error(a.dev, DEV_E_STATE, n, m);
+                        if (src != mine) {
+#pragma unroll
+                            for (int k = 0; k < NV; ++k) mine[k] = r[k];
+                        }
+                    } else {
+                        uint4 pw[P / 16];
+                        read_payload_swizzled<P>(pw, pay + static_cast<size_t>(n % RP) * sh.stage_pay, m);
+                        const uint64_t rk = route_key<P>(x, o, pw);
+                        const uint32_t y = tab[sel * a.tab_stride + x * 8u + o];
+                        r[0].x = y;
+                        r[0].y = r[0].y + 1u;
+                        mix_acc<SB>(r, rk);
+                        uint4 *rp = reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(s) * SB);
+#pragma unroll
+                        for (int k = 0; k < NV; ++k) {
+                            mine[k] = r[k];
+                            rp[k] = r[k];
+                        }
+                        const size_t slot = static_cast<size_t>(n) * K + m;
+                        if (a.effects) {
+                            uint4 e;
+                            e.x = static_cast<uint32_t>(rk);
+                            e.y = static_cast<uint32_t>(rk >> 32);
+                            e.z = s;
+                            e.w = y | (o << 16) | (sel << 24);
+                            __stcs(reinterpret_cast<uint4 *>(a.effects) + slot, e);
+                        }
+                        if (a.state_log) {
+                            uint4 *lp = reinterpret_cast<uint4 *>(a.state_log + slot * SB);
+#pragma unroll
+                            for (int k = 0; k < NV; ++k) __stcs(lp + k, r[k]);
+                        }
+                        odd = static_cast<uint32_t>(rk & 1u);
+                    }
+                }
+            }
+            if (trace) trace[n * 8 + 2] = clock64();
+            if (!early) gather(n + 2u);
+        }
+        // the count of odd keys; the barrier also publishes this step's record
+        // slots and the producer's news, orders the state stores and frees the
+        // slots of step n
+        const uint32_t total = static_cast<uint32_t>(__syncthreads_count(odd));
+        if (trace) trace[n * 8 + 3] = clock64();
+        if (s_ab[n & 1u] != 0u) break;
+        sel = total > K / 2u ? 1u : 0u;
+    }
+    cp_async_wait<0>();
+    if (tid == Kw) {
+        if (n == nst && nst > 0 && a.decisions) a.decisions[nst - 1u] = sel;
+        if (n < nst) {
+            // stopped early: wait (bounded) for the runs and tiles issued so
+            // far (through step n + 5 and n + 3 once the loop ran)
+            const uint32_t w_end = started ? n + RW : RW - 1u, p_end = started ? n + RP : RP - 1u;
+            for (uint32_t j = n; j < w_end && j < nst; ++j) (void)landed_words(j);
+            for (uint32_t j = n; j < p_end && j < nst; ++j) (void)landed_pay(j);
+        }
+    }
+    if (tid == 0 && n == nst) {
+        if (nst > 0) a.dev->sel = sel;
+        a.dev->step = nst;
     }
 }
 
@@ -878,14 +1357,7 @@ __global__ void __launch_bounds__(512, 1)
         s_pending |= 1u << st;
         s_pend_step[st] = j;
     };
-    auto wait_stage = [&](uint32_t st, uint32_t parity) -> bool {
-        const uint64_t t0 = globaltimer_ns();
-        uint32_t spins = 0;
-        while (!mbar_try_wait(&bar[st], parity)) {
-            if ((++spins & 255u) == 0u && globaltimer_ns() - t0 > limit) return false;
-        }
-        return true;
-    };
+    auto wait_stage = [&](uint32_t st, uint32_t parity) -> bool { return mbar_wait_bounded(&bar[st], parity, limit); };
     auto give_up = [&](uint32_t n) {
         latch_error(a.dev, DEV_E_TIMEOUT, n, blockIdx.x);
         atomicExch(&a.dev->abort, 1u);
@@ -1033,7 +1505,7 @@ __global__ void __launch_bounds__(512, 1)
             if (single) {
                 s_sel = total > a.K / 2u ? 1u : 0u;
             } else {
-                const uint64_t t0 = globaltimer_ns();
+                uint64_t t0 = 0;
                 unsigned long long w;
                 uint32_t spins = 0;
                 for (;;) {
@@ -1044,7 +1516,7 @@ __global__ void __launch_bounds__(512, 1)
                             s_abort = 1;
                             break;
                         }
-                        if (globaltimer_ns() - t0 > limit) {
+                        if (timed_out(t0, limit)) {
                             give_up(un);
                             break;
                         }
@@ -1241,7 +1713,7 @@ __global__ void __launch_bounds__(512, 1)
     };
     auto wait_count = [&](uint32_t k, uint32_t *low_prev) -> uint32_t {
         const uint32_t target = (k / 4u + 1u) * G;
-        const uint64_t t0 = globaltimer_ns();
+        uint64_t t0 = 0;
         uint32_t spins = 0, low = 0;
         for (;;) {
             const uint32_t hi = ld_relaxed_hi(&a.dev->slot4[k & 3u], &low);
@@ -1252,7 +1724,7 @@ __global__ void __launch_bounds__(512, 1)
                     s_abort = 1;
                     break;
                 }
-                if (globaltimer_ns() - t0 > limit) {
+                if (timed_out(t0, limit)) {
                     latch_error(a.dev, DEV_E_TIMEOUT, k, b);
                     atomicExch(&a.dev->abort, 1u);
                     s_abort = 1;
@@ -1689,6 +2161,96 @@ cudaError_t launch_chain_grid_tma(const StepArgs &a, int SB, int P, int grid, ui
     TmaShape shc = sh;
     void *args[] = {&map, &aa, &shc};
     return cudaLaunchCooperativeKernel(grid_tma_fn(SB, P), dim3(grid), dim3(threads), args, smem, s);
+}
+
+namespace {
+const void *link_fn_rt(int SB, int P, bool prod) {
+    return dispatch(SB, P, [&](auto b, auto q) {
+        constexpr int B = decltype(b)::value, Q = decltype(q)::value;
+        return prod ? reinterpret_cast<const void *>(&k_chain_cta_prod<B, Q>)
+                    : reinterpret_cast<const void *>(&k_chain_cta_link<B, Q>);
+    });
+}
+size_t link_smem(const LinkShape &sh, uint32_t K, int SB, uint32_t tab_stride) {
+    const size_t Kp = (K + 3u) & ~3u;
+    if (sh.prod)
+        return 1024 + kProdRP * static_cast<size_t>(sh.stage_pay) + kProdRR * static_cast<size_t>(K) * SB +
+               kProdRW * 3ull * K * 4 + 2ull * tab_stride;
+    return 1024 + kLinkRP * static_cast<size_t>(sh.stage_pay) + kLinkRR * Kp * SB + 2ull * kLinkRI * Kp * 4 +
+           kLinkRP * Kp * 4 + 2ull * tab_stride;
+}
+}  // namespace
+
+bool chain_cta_link_plan(int SB, int P, uint32_t K, uint64_t n_sessions, uint32_t tab_stride, bool allow_prod,
+                         size_t *smem, void *shape_out) {
+    if (K == 0 || K > 512u || n_sessions > 0xFFFFFFFFull) return false;
+    const size_t cap = static_cast<size_t>(max_optin_smem());
+    LinkShape sh{};
+    if (allow_prod && K % 8u == 0u && encode_fn()) {
+        sh.prod = 1;
+        sh.n_boxes = K <= 256u ? 1u : 2u;
+        sh.box_rows = (((K + sh.n_boxes - 1u) / sh.n_boxes) + 7u) & ~7u;
+        sh.stage_pay = ((sh.n_boxes * sh.box_rows * static_cast<uint32_t>(P)) + 1023u) & ~1023u;
+        const size_t bytes = link_smem(sh, K, SB, tab_stride);
+        if (bytes <= cap) {
+            *smem = bytes;
+            *static_cast<LinkShape *>(shape_out) = sh;
+            return true;
+        }
+    }
+    sh = LinkShape{};
+    const uint32_t Kp = (K + 3u) & ~3u;
+    sh.stage_pay = ((Kp * static_cast<uint32_t>(P)) + 1023u) & ~1023u;
+    const size_t bytes = link_smem(sh, K, SB, tab_stride);
+    if (bytes > cap) return false;
+    *smem = bytes;
+    *static_cast<LinkShape *>(shape_out) = sh;
+    return true;
+}
+
+cudaError_t launch_link(const StepArgs &a, uint32_t *lnk, cudaStream_t s) {
+    int dev = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    const uint32_t cap = static_cast<uint32_t>(sms) * 4u;
+    const uint32_t grid = a.n_sets < cap ? a.n_sets : cap;
+    const uint32_t threads = a.K >= 512u ? 512u : ((a.K + 31u) / 32u) * 32u;
+    k_link<<<grid ? grid : 1u, threads ? threads : 32u, 0, s>>>(a.idx, a.n_sets, a.K, a.n_sessions, lnk);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_chain_cta_link(const StepArgs &a, int SB, int P, size_t smem, const void *shape,
+                                  const uint32_t *lnk, cudaStream_t s) {
+    const LinkShape &sh = *static_cast<const LinkShape *>(shape);
+    const void *fn = link_fn_rt(SB, P, sh.prod != 0u);
+    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    StepArgs aa = a;
+    const uint32_t *l = lnk;
+    LinkShape shc = sh;
+    const uint32_t member_threads = ((a.K + 31u) / 32u) * 32u;
+    if (!sh.prod) {
+        void *args[] = {&aa, &l, &shc};
+        return cudaLaunchKernel(fn, dim3(1), dim3(member_threads), args, smem, s);
+    }
+    EncodeTiled enc = encode_fn();
+    if (!enc) return cudaErrorNotSupported;
+    alignas(64) CUtensorMap map;
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(P), static_cast<cuuint64_t>(a.n_sets) * a.K};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(P)};
+    const cuuint32_t box[2] = {static_cast<cuuint32_t>(P), sh.box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUtensorMapSwizzle swz = P == 128 ? CU_TENSOR_MAP_SWIZZLE_128B
+                                   : P == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                             : CU_TENSOR_MAP_SWIZZLE_32B;
+    CUresult r = enc(&map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t *>(a.payload), dims, strides, box,
+                     estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    void *args[] = {&map, &aa, &l, &shc};
+    return cudaLaunchKernel(fn, dim3(1), dim3(member_threads + 32u), args, smem, s);
 }
 
 static const void *split_fn(int SB, int P) {

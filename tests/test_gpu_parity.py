@@ -220,7 +220,7 @@ def test_grid_barrier_wait_is_bounded_every_grid_kernel(g, rc, monkeypatch, kern
         rc.rc_free(ctx)
 
 
-@pytest.mark.parametrize("kernel", ["owned", "split", "plain"])
+@pytest.mark.parametrize("kernel", ["owned", "split", "prod", "link", "plain"])
 @pytest.mark.parametrize("P", [32, 64, 128])
 @pytest.mark.parametrize("K,N", [(8, 9), (64, 67), (64, 128), (256, 259), (256, 512), (496, 1000), (512, 513),
                                  (100, 300), (256, 1 << 20)])
@@ -229,6 +229,8 @@ def test_small_cohort_repeated_sessions(g, rc, monkeypatch, kernel, P, K, N):
     persistent kernel must see the records the previous step wrote."""
     monkeypatch.setenv("RC_OWNED", "1" if kernel == "owned" else "0")
     monkeypatch.setenv("RC_SPLIT", "1" if kernel == "split" else "0")
+    monkeypatch.setenv("RC_NO_PIPE", "1" if kernel == "plain" else "0")
+    monkeypatch.setenv("RC_NO_PROD", "1" if kernel == "link" else "0")
     tables, state0, outc, pay, idx = _inputs(60 + K % 13 + P, K, 64, 16, P, 40, N=N)
     n = 40
     want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=1)
@@ -246,3 +248,37 @@ def test_single_cta_identity_sessions(g, rc, monkeypatch, pipe, SB, P, K):
     want = g.run_oracle(tables, state0, outc, pay, idx, n)
     got = g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K)
     g.assert_same(got, want, f"identity pipe={pipe} SB={SB} P={P} K={K}")
+
+
+@pytest.mark.parametrize("n_sets", [1, 2, 3, 7])
+@pytest.mark.parametrize("SB,P,K,extra,want_launches", [(16, 64, 256, 0, 2), (16, 64, 256, 1, 2), (16, 32, 7, 2, 2),
+                                                   (64, 64, 256, 1, 2), (16, 128, 300, 3, 2), (64, 32, 33, 0, 2),
+                                                   (16, 64, 264, 9, 2), (16, 64, 512, 5, 2), (64, 128, 512, 1, 1)])
+def test_linked_single_cta_ring_wraps(g, rc, SB, P, K, extra, want_launches, n_sets):
+    """The single-CTA chain that gathers records two steps early: cohorts drawn
+    from N = K + extra sessions, so nearly every session recurs in the next two
+    steps at another position, and a ring of 1, 2, 3 or 7 cohorts, so links wrap
+    (with one cohort every member follows itself).  K a multiple of 8 takes the
+    producer-warp form (payload tiles: one, or two for K > 256), other K the
+    per-thread-copy form.  Both launches (link pass and
+    chain) are counted where the kernel applies; 512 members with 64-byte
+    records and 128-byte payloads do not fit its rings and take the plain
+    single-CTA kernel (one launch)."""
+    import torch
+    S = 256 if SB == 64 else 64
+    N = K + extra
+    tables, state0, outc, pay, idx = _inputs(90 + n_sets + K % 7, K, S, SB, P, n_sets, N=N)
+    n = 13
+    want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=1)
+    got = g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K, sel0=1)
+    g.assert_same(got, want, f"linked n_sets={n_sets} SB={SB} P={P} K={K} N={N}")
+    ctx = rc.rc_init(S, tables, SB, P, K, N, torch.cuda.current_stream())
+    try:
+        state = g.dev(state0.copy())
+        ev = rc.make_events(g.dev(outc), g.dev(pay), g.dev(idx), n_sets=n_sets)
+        dec = torch.zeros(n, dtype=torch.int32, device="cuda")
+        rc.rc_chain(ctx, n, rc.RC_MECH_RESIDENT_PERSIST, state, ev, K, dec)
+        _, launches = rc.rc_last_chain_stats(ctx)
+        assert launches == want_launches
+    finally:
+        rc.rc_free(ctx)
