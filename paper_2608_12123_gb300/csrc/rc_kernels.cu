@@ -540,10 +540,13 @@ __global__ void __launch_bounds__(1024, 1) k_chain_cta_ident(StepArgs a) {
 
 // ---------------------------------------------------------------------------
 // Persistent chain, cooperative grid (any K): each CTA owns a grid-stride
-// slice of members.  Per step, thread 0 of each CTA adds (1 << 32 | odd
-// count) to the step's barrier word with release semantics and spins with
-// acquire loads until all CTAs have arrived; the low half is then the full
-// odd count, so every CTA derives the decision itself.  Three rotating words:
+// slice of members.  Per step, after a block barrier, thread 0 of each CTA
+// adds (1 << 32 | odd count) to the step's barrier word with release
+// semantics and spins with acquire loads until all CTAs have arrived, then a
+// block barrier hands the result on: the release is cumulative over the
+// block's stores (ordered before it by the first block barrier) and the
+// acquire over the block's later loads, so no separate fence is needed.  The
+// low half is then the full odd count, so every CTA derives the decision.  Three rotating words:
 // CTA 0 clears word (n+1) % 3 before arriving at step n, when no CTA can still
 // be reading it.  Spins are bounded by dev->wait_ns; on expiry the CTA latches
 // RC_E_TIMEOUT, raises dev->abort and returns, and the others follow.
@@ -584,7 +587,6 @@ __global__ void __launch_bounds__(kGridThreads) k_chain_grid(StepArgs a) {
             if (blockIdx.x == 0) {
                 a.dev->slot[(n + 1u) % 3u] = 0ull;
             }
-            __threadfence();
             const bool skip = (n == 0 && blockIdx.x == 1 && ld_volatile_u32(&a.dev->skip_arrival) != 0u);
             if (!skip) red_release_add_u64(word, (1ull << 32) | c);
             uint64_t t0 = 0;
@@ -606,7 +608,6 @@ __global__ void __launch_bounds__(kGridThreads) k_chain_grid(StepArgs a) {
                     }
                 }
             }
-            __threadfence();
             const uint32_t d = (static_cast<uint32_t>(w & 0xffffffffull) > a.K / 2u) ? 1u : 0u;
             s_sel = d;
             if (blockIdx.x == 0 && a.decisions && !s_abort) a.decisions[n] = d;
@@ -657,9 +658,101 @@ __device__ __forceinline__ void read_payload_swizzled(uint4 (&pw)[P / 16], const
     }
 }
 
+// One step of the members [m0, m0 + cnt) of a TMA-fed CTA whose records are
+// 64 bytes or more, one member per thread (cnt <= blockDim.x).  The records are
+// gathered and stored warp-cooperatively (NV lanes per record, chunks staged in
+// shared memory), so a copy instruction of a warp touches 32 / NV records
+// rather than one chunk of 32 records.  Same results and error latching as
+// transition(); returns this thread's odd-key count.
+template <int SB, int P>
+__device__ __forceinline__ uint32_t coop_transition(const StepArgs &a, const uint32_t *idx_st, const uint32_t *out_st,
+                                                    const uint8_t *pay_st, uint4 *rec_st, uint32_t cnt, uint32_t m0,
+                                                    const uint8_t *tab, uint32_t sel, uint32_t n, uint64_t keep) {
+    constexpr uint32_t NV = SB / 16;
+    constexpr uint32_t RPI = 32u / NV;
+    const uint32_t tid = threadIdx.x;
+    const uint32_t lane = tid & 31u, wbase = tid & ~31u;
+    const uint32_t c = lane % NV;
+    auto session_of = [&](uint32_t t) { return a.idx ? idx_st[t] : m0 + t; };
+    // gather the warp's records (a copy whose stage slot would leave the
+    // block's stage is refused and latched: the stage holds blockDim.x records)
+#pragma unroll
+    for (uint32_t k = 0; k < NV; ++k) {
+        const uint32_t t = wbase + k * RPI + lane / NV;
+        if (t < cnt) {
+            const uint32_t s = session_of(t);
+            const uint32_t slot = pay_chunk<SB>(t, c);
+            if (slot >= blockDim.x * NV)
+                latch_error(a.dev, DEV_E_INDEX, n, 0xFFFFFF00u | t);
+            else if (s < a.n_sessions)
+                cp_async16(rec_st + slot, reinterpret_cast<const uint4 *>(a.state + static_cast<size_t>(s) * SB) + c);
+        }
+    }
+    cp_async_commit();
+    cp_async_wait<0>();
+    __syncwarp();
+    uint32_t odd = 0, updated = 0;
+    if (tid < cnt) {
+        const uint32_t m = m0 + tid;
+        const uint32_t s = session_of(tid);
+        const uint32_t o = out_st[tid];
+        if (s >= a.n_sessions) {
+            latch_error(a.dev, DEV_E_INDEX, n, m);
+        } else {
+            uint4 r[NV];
+#pragma unroll
+            for (uint32_t k = 0; k < NV; ++k) r[k] = rec_st[pay_chunk<SB>(tid, k)];
+            const uint32_t x = r[0].x;
+            if (x >= a.S || o >= 8u) {
+                latch_error(a.dev, DEV_E_STATE, n, m);
+            } else {
+                uint4 pw[P / 16];
+                read_payload_swizzled<P>(pw, pay_st, tid);
+                const uint64_t rk = route_key<P>(x, o, pw);
+                const uint32_t y = tab[x * 8u + o];
+                r[0].x = y;
+                r[0].y = r[0].y + 1u;
+                mix_acc<SB>(r, rk);
+#pragma unroll
+                for (uint32_t k = 0; k < NV; ++k) rec_st[pay_chunk<SB>(tid, k)] = r[k];
+                const size_t slot = static_cast<size_t>(n) * a.K + m;
+                if (a.effects) {
+                    uint4 e;
+                    e.x = static_cast<uint32_t>(rk);
+                    e.y = static_cast<uint32_t>(rk >> 32);
+                    e.z = s;
+                    e.w = y | (o << 16) | (sel << 24);
+                    __stcs(reinterpret_cast<uint4 *>(a.effects) + slot, e);
+                }
+                if (a.state_log) {
+                    uint4 *lp = reinterpret_cast<uint4 *>(a.state_log + slot * SB);
+#pragma unroll
+                    for (uint32_t k = 0; k < NV; ++k) __stcs(lp + k, r[k]);
+                }
+                odd = static_cast<uint32_t>(rk & 1u);
+                updated = 1;
+            }
+        }
+    }
+    // store the warp's updated records
+    const uint32_t upd = __ballot_sync(0xffffffffu, updated);
+    __syncwarp();
+#pragma unroll
+    for (uint32_t k = 0; k < NV; ++k) {
+        const uint32_t q = k * RPI + lane / NV;
+        const uint32_t t = wbase + q;
+        if ((upd >> q) & 1u) {
+            const uint32_t s = session_of(t);
+            st_hint(reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(s) * SB) + c, rec_st[pay_chunk<SB>(t, c)], keep);
+        }
+    }
+    return odd;
+}
+
 template <int SB, int P>
 __global__ void __launch_bounds__(512, 1)
     k_chain_grid_tma(const __grid_constant__ CUtensorMap tmap, StepArgs a, TmaShape sh) {
+    constexpr int NV = SB / 16;
     extern __shared__ uint8_t dsm_raw[];
     __shared__ __align__(8) uint64_t bar[2];
     __shared__ uint32_t warp_odd[16];
@@ -669,6 +762,9 @@ __global__ void __launch_bounds__(512, 1)
     uint8_t *const base = dsm_raw + (((raw + 1023u) & ~1023u) - raw);
     uint32_t *const words = reinterpret_cast<uint32_t *>(base + 2 * sh.stage_pay);
     uint8_t *const tab = reinterpret_cast<uint8_t *>(words + 4 * sh.stage_words);
+    // 64-byte records: a shared stage of one record per thread (chunks placed
+    // by pay_chunk, so that quarter-warps hit eight bank groups)
+    uint4 *const rec_st = reinterpret_cast<uint4 *>(tab + ((2 * a.tab_stride + 15u) & ~15u));
     auto pay_of = [&](uint32_t st) { return base + st * sh.stage_pay; };
     auto out_of = [&](uint32_t st) { return words + st * sh.stage_words; };
     auto idx_of = [&](uint32_t st) { return words + (2u + st) * sh.stage_words; };
@@ -733,12 +829,17 @@ __global__ void __launch_bounds__(512, 1)
         __syncthreads();
         if (s_abort) break;
         if (trace) trace[n * 8 + 1] = clock64();
-        for (uint32_t t = tid; t < cnt; t += blockDim.x) {
-            Event<P> ev;
-            ev.s = a.idx ? idx_of(st)[t] : m0 + t;
-            ev.o = out_of(st)[t];
-            read_payload_swizzled<P>(ev.pw, pay_of(st), t);
-            odd += transition<SB, P, true, true>(a, ev, tab + sel * a.tab_stride, sel, n, m0 + t, keep_pol);
+        if (NV >= 2 && cnt <= blockDim.x) {
+            odd = coop_transition<SB, P>(a, idx_of(st), out_of(st), pay_of(st), rec_st, cnt, m0,
+                                         tab + sel * a.tab_stride, sel, n, keep_pol);
+        } else {
+            for (uint32_t t = tid; t < cnt; t += blockDim.x) {
+                Event<P> ev;
+                ev.s = a.idx ? idx_of(st)[t] : m0 + t;
+                ev.o = out_of(st)[t];
+                read_payload_swizzled<P>(ev.pw, pay_of(st), t);
+                odd += transition<SB, P, true, true>(a, ev, tab + sel * a.tab_stride, sel, n, m0 + t, keep_pol);
+            }
         }
         uint32_t v = odd;
 #pragma unroll
@@ -751,7 +852,6 @@ __global__ void __launch_bounds__(512, 1)
             for (uint32_t w = 0; w < (blockDim.x + 31u) / 32u; ++w) c += warp_odd[w];
             unsigned long long *word = &a.dev->slot[n % 3u];
             if (blockIdx.x == 0) a.dev->slot[(n + 1u) % 3u] = 0ull;
-            __threadfence();
             const bool skip = (n == 0 && blockIdx.x == 1 && ld_volatile_u32(&a.dev->skip_arrival) != 0u);
             if (!skip) red_release_add_u64(word, (1ull << 32) | c);
             if (trace) trace[n * 8 + 3] = clock64();
@@ -782,7 +882,6 @@ __global__ void __launch_bounds__(512, 1)
                     }
                 }
             }
-            __threadfence();
             if (trace) trace[n * 8 + 5] = clock64();
             const uint32_t d = (static_cast<uint32_t>(w & 0xffffffffull) > a.K / 2u) ? 1u : 0u;
             s_sel = d;
@@ -1695,20 +1794,36 @@ __global__ void __launch_bounds__(512, 1)
         r.o = __ldg(perm_o + e);
         r.valid = v ? 1u : 0u;
     };
-    auto stage_row = [&](uint32_t j, const Routed &r) {
-        if (!r.valid) return;
-        const uint4 *src =
-            reinterpret_cast<const uint4 *>(a.payload + (static_cast<size_t>(j % a.n_sets) * a.K + r.m) * P);
+    // The warp's rows and records are copied warp-cooperatively: NC (NV) lanes
+    // take the 16-byte chunks of one payload row (record), so one copy
+    // instruction of the warp touches 32 / NC whole rows instead of a chunk of
+    // 32 rows; each lane learns the row's member or session by a shuffle.
+    const uint32_t lane = tid & 31u, wbase = tid & ~31u;
+    auto stage_row = [&](uint32_t j, const Routed &r) {  // all lanes of the warp
+        constexpr uint32_t RPI = 32u / NC;
         uint4 *dst = pay + static_cast<size_t>(j & 1u) * T * NC;
+        const size_t set0 = static_cast<size_t>(j % a.n_sets) * a.K;
+        const uint32_t c = lane % NC;
 #pragma unroll
-        for (uint32_t k = 0; k < NC; ++k) cp_async16(dst + pay_chunk<P>(tid, k), src + k);
+        for (uint32_t k = 0; k < NC; ++k) {
+            const uint32_t from = k * RPI + lane / NC;
+            const uint32_t m = __shfl_sync(0xffffffffu, r.m, from);
+            const uint32_t v = __shfl_sync(0xffffffffu, r.valid, from);
+            if (v) cp_async16(dst + pay_chunk<P>(wbase + from, c), reinterpret_cast<const uint4 *>(a.payload + (set0 + m) * P) + c);
+        }
     };
-    auto stage_record = [&](const Routed &r) {
+    auto stage_record = [&](const Routed &r) {  // all lanes of the warp
         if constexpr (!RES) {
-            if (!r.valid) return;
-            const uint4 *rp = reinterpret_cast<const uint4 *>(a.state + static_cast<size_t>(r.s) * SB);
+            constexpr uint32_t RPI = 32u / NV;
+            const uint32_t c = lane % NV;
 #pragma unroll
-            for (int k = 0; k < NV; ++k) cp_async16(rec_st + static_cast<size_t>(tid) * NV + k, rp + k);
+            for (uint32_t k = 0; k < static_cast<uint32_t>(NV); ++k) {
+                const uint32_t from = k * RPI + lane / NV;
+                const uint32_t s2 = __shfl_sync(0xffffffffu, r.s, from);
+                const uint32_t v = __shfl_sync(0xffffffffu, r.valid, from);
+                if (v) cp_async16(rec_st + static_cast<size_t>(wbase + from) * NV + c,
+                                  reinterpret_cast<const uint4 *>(a.state + static_cast<size_t>(s2) * SB) + c);
+            }
         }
     };
     auto wait_count = [&](uint32_t k, uint32_t *low_prev) -> uint32_t {
@@ -1759,7 +1874,8 @@ __global__ void __launch_bounds__(512, 1)
         cp_async_commit();
         stage_row(n + 1u, r1);      // rows of step n + 1
         cp_async_commit();
-        cp_async_wait<2>();         // this thread's row of step n is here
+        cp_async_wait<2>();         // this lane's row copies of step n are here
+        __syncwarp();               // and so are the other lanes' (the warp's rows)
         if (trace) trace[n * 8 + 1] = clock64();
         const size_t e0 = static_cast<size_t>(n % a.n_sets) * a.K;
         const uint32_t cnt0 = hi0 - lo0;
@@ -1819,10 +1935,14 @@ __global__ void __launch_bounds__(512, 1)
         __syncthreads();
         if (s_abort) break;
         if (n > 0) sel = s_sel;
-        cp_async_wait<1>();  // this thread's record of step n is here
+        cp_async_wait<1>();  // the warp's records of step n are here
+        __syncwarp();
         if (trace) trace[n * 8 + 6] = clock64();
         // --- next state, record and effect (body chosen by the decision of step n - 1) ---
-        auto finish = [&](uint32_t s2, uint32_t m2, uint32_t o2, uint32_t x2, uint64_t rk2, uint4 (&rr)[NV]) {
+        // coop: the record goes back to this thread's shared stage, and the warp
+        // stores the stages cooperatively below
+        auto finish = [&](uint32_t s2, uint32_t m2, uint32_t o2, uint32_t x2, uint64_t rk2, uint4 (&rr)[NV],
+                          bool coop) {
             const uint32_t y = tab[sel * a.tab_stride + x2 * 8u + o2];
             rr[0].x = y;
             rr[0].y = rr[0].y + 1u;
@@ -1833,9 +1953,14 @@ __global__ void __launch_bounds__(512, 1)
                 for (int k = 0; k < NV; ++k) owned_rec[static_cast<size_t>(ls) * NV + k] = rr[k];
             } else {
                 owned[ls] = static_cast<uint8_t>(y);
-                uint4 *rp = reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(s2) * SB);
+                if (coop) {
 #pragma unroll
-                for (int k = 0; k < NV; ++k) rp[k] = rr[k];
+                    for (int k = 0; k < NV; ++k) rec_st[static_cast<size_t>(tid) * NV + k] = rr[k];
+                } else {
+                    uint4 *rp = reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(s2) * SB);
+#pragma unroll
+                    for (int k = 0; k < NV; ++k) rp[k] = rr[k];
+                }
             }
             const size_t slot = static_cast<size_t>(n) * a.K + m2;
             if (a.effects) {
@@ -1861,7 +1986,22 @@ __global__ void __launch_bounds__(512, 1)
 #pragma unroll
                 for (int k = 0; k < NV; ++k) rr[k] = rec_st[static_cast<size_t>(tid) * NV + k];
             }
-            finish(r0.s, r0.m, r0.o, x, rk, rr);
+            finish(r0.s, r0.m, r0.o, x, rk, rr, true);
+        }
+        if constexpr (!RES) {
+            // the warp's updated records, NV lanes per record
+            __syncwarp();
+            constexpr uint32_t RPI = 32u / NV;
+            const uint32_t c = lane % NV;
+#pragma unroll
+            for (uint32_t k = 0; k < static_cast<uint32_t>(NV); ++k) {
+                const uint32_t from = k * RPI + lane / NV;
+                const uint32_t s2 = __shfl_sync(0xffffffffu, r0.s, from);
+                const uint32_t v = __shfl_sync(0xffffffffu, ok ? 1u : 0u, from);
+                if (v)
+                    reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(s2) * SB)[c] =
+                        rec_st[static_cast<size_t>(wbase + from) * NV + c];
+            }
         }
         for (uint32_t p = tid + T; p < cnt0; p += T) {
             const size_t e = e0 + lo0 + p;
@@ -1883,7 +2023,7 @@ __global__ void __launch_bounds__(512, 1)
             const uint4 *src = reinterpret_cast<const uint4 *>(a.payload + (e0 + m2) * P);
 #pragma unroll
             for (uint32_t k = 0; k < NC; ++k) pw[k] = __ldg(src + k);
-            finish(s2, m2, o2, x2, route_key<P>(x2, o2, pw), rr);
+            finish(s2, m2, o2, x2, route_key<P>(x2, o2, pw), rr, false);
         }
         __syncthreads();  // owned state updated before the next step reads it; stages free
         if (trace) trace[n * 8 + 7] = clock64();
@@ -2120,7 +2260,9 @@ bool chain_grid_tma_plan(int SB, int P, uint32_t K, uint32_t tab_stride, int *gr
     sh.box_rows = (((sh.chunk + sh.n_boxes - 1u) / sh.n_boxes) + 7u) & ~7u;
     sh.stage_pay = ((sh.n_boxes * sh.box_rows * static_cast<uint32_t>(P)) + 1023u) & ~1023u;
     sh.stage_words = (sh.chunk + 3u) & ~3u;
-    const size_t bytes = tma_smem_bytes(sh, tab_stride);
+    const uint32_t thr = sh.chunk >= 512u ? 512u : ((sh.chunk + 31u) / 32u) * 32u;
+    const size_t rec_stage = SB >= 64 ? static_cast<size_t>(thr) * SB + 16 : 0;
+    const size_t bytes = tma_smem_bytes(sh, tab_stride) + rec_stage;
     if (bytes + 2048 > static_cast<size_t>(max_optin)) return false;
     const void *fn = grid_tma_fn(SB, P);
     if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes)) !=
@@ -2128,7 +2270,6 @@ bool chain_grid_tma_plan(int SB, int P, uint32_t K, uint32_t tab_stride, int *gr
         cudaGetLastError();
         return false;
     }
-    const uint32_t thr = sh.chunk >= 512u ? 512u : ((sh.chunk + 31u) / 32u) * 32u;
     int per_sm = 0;
     if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, static_cast<int>(thr), bytes) != cudaSuccess ||
         per_sm < 1 || static_cast<long long>(per_sm) * sms < g)
