@@ -339,7 +339,7 @@ def native(args):
 
         alg_bytes = H * K * BYTES_PER_TRANSITION_C2
         ach = alg_bytes / (step_ms * 1e-3) / 1e9
-        traffic = ncu_traffic("k_chain_cta<16,64>", H * K)
+        traffic = ncu_traffic("k_chain_cta_prod<16,64>", H * K)
         out.update({
             "metric": METRIC, "value": round(value, 4), "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(step_ms, 4), "higher_is_better": False,
@@ -361,7 +361,7 @@ def native(args):
                                 "vs_launch_sync": round(us_inv / floor_probe["launch_sync"], 3)},
             "roofline": {"bound": "hbm", "achieved": round(ach, 3), "peak": hbm_peak, "unit": "GB/s",
                          "frac": round(ach / hbm_peak, 5), "traffic": traffic,
-                         "kernel": "k_chain_cta<16,64> (one launch = 1,000 steps x 256 members)",
+                         "kernel": "k_chain_cta_prod<16,64> (one launch = 1,000 steps x 256 members, after the k_link pass)",
                          "peak_source": f"{peak_src} hbm_gbs",
                          "note": "K=256 steps are latency-bound: see latency_x_floor"},
             "e2e": {"value": round(e2e_us, 4), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
@@ -430,8 +430,8 @@ def large_k(args, rc, torch, stream, hbm_peak, peak_src, flush, world):
         "transitions_per_s": round(world * K * n / (ms * 1e-3), 1),
         "hbm_gbs": round(gbs, 1),
         "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": hbm_peak, "unit": "GB/s",
-                     "frac": round(gbs / hbm_peak, 4), "traffic": ncu_traffic("k_chain_grid_tma<64,128>", K),
-                     "kernel": "k_chain_grid_tma<64,128> (cooperative persistent grid, TMA-fed), per invocation",
+                     "frac": round(gbs / hbm_peak, 4), "traffic": ncu_traffic("k_chain_grid_link<64,128>", K),
+                     "kernel": "k_chain_grid_link<64,128> (cooperative persistent grid split by links, TMA-fed), per invocation",
                      "algorithmic_bytes_per_invocation": alg, "peak_source": f"{peak_src} hbm_gbs (burst)"},
         "l2": "inputs larger than L2 (64 MiB state + 550 MB event ring + 1 GiB effects) and flushed per chain",
         "us_per_invocation_resident": round(us_inv, 4),

@@ -91,6 +91,7 @@ struct rc_ctx {
     bool no_pipe = false;   // RC_NO_PIPE=1 selects the plain single-CTA kernel
     bool no_link = false;   // RC_NO_LINK=1 turns off the linked single-CTA kernels
     bool no_prod = false;   // RC_NO_PROD=1 keeps the linked kernel without a producer warp
+    bool no_grid_link = false;  // RC_NO_GRID_LINK=1 turns off the grid chain split by links
     bool use_split = false;  // RC_SPLIT=1 selects the split-phase chain (slower on GB300 so far)
     bool use_owned = false;  // RC_OWNED=1 selects the session-owned chain
     Buf route_buf;           // session-owned chain: routed member lists
@@ -444,6 +445,21 @@ int run_persist(rc_ctx *c, const rc::StepArgs &a) {
     if (!c->coop) return fail(c, RC_E_UNSUPPORTED, "device lacks cooperative launch");
     RC_CUDA(c, cudaMemsetAsync(c->dev->slot, 0, sizeof(c->dev->slot), c->stream));
     RC_CUDA(c, cudaMemsetAsync(&c->dev->abort, 0, sizeof(uint32_t), c->stream));
+    if (a.idx && !c->no_grid_link) {
+        int grid = 0;
+        uint32_t threads = 0;
+        size_t smem = 0, scratch = 0;
+        alignas(8) unsigned char shape[48];
+        if (rc::chain_grid_link_plan(c->SB, c->P, a.K, c->n_sessions, a.n_sets, c->tab_stride, &grid, &threads, &smem,
+                                     shape, &scratch)) {
+            int rc = ensure(c, c->link_buf, scratch);
+            if (rc != RC_OK) return rc;
+            c->last_launches = 3;  // mark + flag passes, chain
+            RC_CUDA(c, rc::launch_chain_grid_link(a, c->SB, c->P, grid, threads, smem, shape, c->link_buf.p, c->stream));
+            RC_CUDA(c, cudaMemsetAsync(&c->dev->skip_arrival, 0, sizeof(uint32_t), c->stream));
+            return RC_OK;
+        }
+    }
     int grid = 0;
     uint32_t threads = 0;
     size_t smem = 0;
@@ -577,6 +593,8 @@ int rc_init(rc_ctx **out, uint32_t S, const uint8_t *table, uint32_t state_bytes
         c->no_link = z && z[0] == '1';
         const char *q = std::getenv("RC_NO_PROD");
         c->no_prod = q && q[0] == '1';
+        const char *gl = std::getenv("RC_NO_GRID_LINK");
+        c->no_grid_link = gl && gl[0] == '1';
         const char *x = std::getenv("RC_SPLIT");
         c->use_split = x && x[0] == '1';
         const char *y = std::getenv("RC_OWNED");

@@ -1383,6 +1383,350 @@ __global__ void __launch_bounds__(544, 1)
 }
 
 // ---------------------------------------------------------------------------
+// Persistent chain, cooperative grid, split by links (explicit session
+// indices, K a multiple of 8; one CTA per SM, CTA b owns the contiguous
+// members [b*chunk, b*chunk + cnt) as in k_chain_grid_tma).
+//
+// lnk[j][m] is non-zero when member m's session also sits in cohort j - 1
+// (k_mark / k_flag).  Only such a "linked" member of step n + 1 needs the
+// records stored in step n; every other member's record was last stored in
+// step n - 1 or earlier, which the grid barrier of step n - 1 already made
+// visible.  So each step splits in two regions:
+//   A(n)  after the barrier of step n - 1: gather and hash the linked members
+//         of step n; then transition every member of step n with d(n - 1),
+//         store the records (warp-cooperatively, NV lanes per record) and
+//         stage the effects in shared memory;
+//   B(n)  the control thread (lane 0 of the last warp) adds (1 << 32 | odd
+//         count of step n) to the barrier word with release semantics,
+//         stores the effect run of step n with one bulk copy (so the release
+//         does not wait for it), issues the event copies of step n + 2 and
+//         spins for all CTAs; meanwhile the member warps gather and hash the
+//         unlinked members of step n + 1.
+// Step 0 has no earlier step in the launch: all its members count as
+// unlinked.  Every wait is bounded: a CTA that gives up latches
+// RC_E_TIMEOUT, raises dev->abort and leaves after the next block barrier,
+// the control thread first waiting (bounded) for its copies in flight.
+// ---------------------------------------------------------------------------
+struct GridLinkShape {
+    TmaShape t;         // chunk, payload tiles, stage sizes (as k_chain_grid_tma)
+    uint32_t members;   // member threads (a multiple of 32, >= chunk); the control warp follows
+    uint32_t pad[3];
+};
+
+__device__ __forceinline__ void bulk_store(void *gdst, const void *ssrc, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(gdst), "r"(smem_addr(ssrc)),
+                 "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+template <int N>
+__device__ __forceinline__ void bulk_wait_all() {
+    asm volatile("cp.async.bulk.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// Marks, per cohort j of the ring, its sessions in bitmap bits[j] (words of
+// 32 sessions; the caller clears the bitmaps).
+__global__ void k_mark(const uint32_t *idx, uint32_t n_sets, uint32_t K, uint64_t N, uint64_t words_per_set,
+                       uint32_t *bits) {
+    const size_t total = static_cast<size_t>(n_sets) * K;
+    for (size_t e = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < total;
+         e += static_cast<size_t>(gridDim.x) * blockDim.x) {
+        const uint32_t s = idx[e];
+        if (s >= N) continue;
+        const size_t j = e / K;
+        atomicOr(bits + j * words_per_set + (s >> 5), 1u << (s & 31u));
+    }
+}
+
+// lnk[j][m] = 1 when member m's session of cohort j is in cohort j - 1 (mod n_sets).
+__global__ void k_flag(const uint32_t *idx, uint32_t n_sets, uint32_t K, uint64_t N, uint64_t words_per_set,
+                       const uint32_t *bits, uint32_t *lnk) {
+    const size_t total = static_cast<size_t>(n_sets) * K;
+    for (size_t e = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < total;
+         e += static_cast<size_t>(gridDim.x) * blockDim.x) {
+        const uint32_t s = idx[e];
+        const size_t j = e / K;
+        const size_t jp = (j + n_sets - 1) % n_sets;
+        uint32_t l = 0;
+        if (s < N) l = (bits[jp * words_per_set + (s >> 5)] >> (s & 31u)) & 1u;
+        lnk[e] = l;
+    }
+}
+
+template <int SB, int P>
+__global__ void __launch_bounds__(544, 1)
+    k_chain_grid_link(const __grid_constant__ CUtensorMap tmap, StepArgs a, const uint32_t *lnk, GridLinkShape gs) {
+    constexpr uint32_t NV = SB / 16;
+    constexpr uint32_t RPI = 32u / NV;
+    const TmaShape sh = gs.t;
+    extern __shared__ uint8_t dsm_raw[];
+    __shared__ __align__(8) uint64_t bar[2];
+    __shared__ uint32_t warp_odd[17];
+    __shared__ uint32_t s_sel, s_rej;
+    __shared__ uint32_t s_upd[17];  // per member warp: which lanes transitioned this step
+    __shared__ uint32_t s_ab[2];  // [0]: raised in region A, read after its barrier; [1]: region B
+    // layout: [pay 0][pay 1][out 0|1][idx 0|1][lnk 0|1][tables][records 0|1][effects 0|1]
+    const uint32_t raw = smem_addr(dsm_raw);
+    uint8_t *const base = dsm_raw + (((raw + 1023u) & ~1023u) - raw);
+    uint32_t *const words = reinterpret_cast<uint32_t *>(base + 2 * sh.stage_pay);
+    uint8_t *const tab = reinterpret_cast<uint8_t *>(words + 6 * sh.stage_words);
+    uint4 *const recs = reinterpret_cast<uint4 *>(tab + ((2 * a.tab_stride + 15u) & ~15u));
+    uint4 *const effs = recs + 2ull * sh.chunk * NV;
+    auto pay_of = [&](uint32_t st) { return base + st * sh.stage_pay; };
+    auto out_of = [&](uint32_t st) { return words + st * sh.stage_words; };
+    auto idx_of = [&](uint32_t st) { return words + (2u + st) * sh.stage_words; };
+    auto lnk_of = [&](uint32_t st) { return words + (4u + st) * sh.stage_words; };
+    auto rec_of = [&](uint32_t st) { return recs + static_cast<size_t>(st) * sh.chunk * NV; };
+    auto eff_of = [&](uint32_t st) { return effs + static_cast<size_t>(st) * sh.chunk; };
+
+    const uint32_t tid = threadIdx.x;
+    const bool ctl = tid == gs.members;
+    const bool member = tid < gs.members;
+    const uint32_t lane = tid & 31u, wbase = tid & ~31u;
+    const uint32_t G = gridDim.x;
+    const uint32_t m0 = blockIdx.x * sh.chunk;
+    const uint32_t cnt = m0 < a.K ? min(sh.chunk, a.K - m0) : 0u;
+    const uint32_t nst = a.n_steps;
+    const uint64_t limit = a.dev->wait_ns;
+    const uint64_t stream_pol = policy_evict_first();
+    const uint64_t keep_pol = policy_evict_last();
+    // profiling: the control thread and member thread 0 of the first and last CTA
+    long long *trace = nullptr;
+    if (a.trace && (tid == 0 || ctl) && (blockIdx.x == 0 || blockIdx.x == G - 1))
+        trace = a.trace + (blockIdx.x == 0 ? 0 : static_cast<size_t>(nst) * 8) + (ctl ? 0 : 4);
+
+    uint32_t issued = 0;  // control thread: steps [0, issued) have had their events issued
+    auto issue = [&](uint32_t j) {  // control thread: events of step j into stage j & 1
+        issued = j + 1u;
+        const uint32_t st = j & 1u;
+        const uint32_t row0 = (j % a.n_sets) * a.K + m0;
+        mbar_arrive_expect_tx(&bar[st], sh.n_boxes * sh.box_rows * P + cnt * 12u);
+        for (uint32_t b = 0; b < sh.n_boxes; ++b)
+            tma_load_2d_hint(pay_of(st) + b * sh.box_rows * P, &tmap, 0,
+                             static_cast<int32_t>(row0 + b * sh.box_rows), &bar[st], stream_pol);
+        bulk_load_hint(out_of(st), a.outcome + row0, cnt * 4u, &bar[st], stream_pol);
+        bulk_load_hint(idx_of(st), a.idx + row0, cnt * 4u, &bar[st], stream_pol);
+        bulk_load_hint(lnk_of(st), lnk + row0, cnt * 4u, &bar[st], stream_pol);
+    };
+    auto linked = [&](uint32_t j, uint32_t t) { return j > 0u && lnk_of(j & 1u)[t] != 0u; };
+    // member warps: gather the records of step j's members of this warp whose
+    // linked flag equals want, NV lanes per record
+    auto gather = [&](uint32_t j, bool want) {
+        const uint32_t st = j & 1u;
+        const uint32_t c = lane % NV;
+#pragma unroll
+        for (uint32_t k = 0; k < NV; ++k) {
+            const uint32_t t = wbase + k * RPI + lane / NV;
+            if (t < cnt && linked(j, t) == want) {
+                const uint32_t s = idx_of(st)[t];
+                if (s < a.n_sessions)
+                    cp_async16(rec_of(st) + pay_chunk<SB>(t, c),
+                               reinterpret_cast<const uint4 *>(a.state + static_cast<size_t>(s) * SB) + c);
+            }
+        }
+        cp_async_commit();
+        cp_async_wait<0>();
+        __syncwarp();
+    };
+    // this thread's member of step j (when its linked flag equals want): route key
+    uint64_t rk = 0;
+    uint32_t ok = 0, odd = 0;
+    auto key = [&](uint32_t j, bool want) {
+        if (tid >= cnt || linked(j, tid) != want) return;
+        const uint32_t st = j & 1u;
+        const uint32_t s = idx_of(st)[tid], o = out_of(st)[tid];
+        ok = 0;
+        odd = 0;
+        if (s >= a.n_sessions) {
+            latch_error(a.dev, DEV_E_INDEX, j, m0 + tid);
+            return;
+        }
+        const uint32_t x = rec_of(st)[pay_chunk<SB>(tid, 0)].x;
+        if (x >= a.S || o >= 8u) {
+            latch_error(a.dev, DEV_E_STATE, j, m0 + tid);
+            return;
+        }
+        uint4 pw[P / 16];
+        read_payload_swizzled<P>(pw, pay_of(st), tid);
+        rk = route_key<P>(x, o, pw);
+        odd = static_cast<uint32_t>(rk & 1u);
+        ok = 1;
+    };
+
+    if (ctl) {
+        mbar_init(&bar[0], 1);
+        mbar_init(&bar[1], 1);
+        fence_mbar_init();
+        s_sel = ld_volatile_u32(&a.dev->sel) & 1u;
+        s_ab[0] = 0;
+        s_ab[1] = 0;
+        s_rej = 0;
+    }
+    stage_tables(tab, a.tables, a.tab_stride, 2, 0);
+    __syncthreads();
+    if (ctl && cnt > 0) {
+        if (nst > 0) issue(0);
+        if (nst > 1) issue(1);
+    }
+    uint32_t sel = s_sel;
+    // prologue: step 0 (all members unlinked) gathered and hashed
+    if (member && cnt > 0 && nst > 0) {
+        if (!mbar_wait_bounded(&bar[0], 0u, limit)) {
+            latch_error(a.dev, DEV_E_TIMEOUT, 0, blockIdx.x);
+            s_ab[1] = 1;
+        } else {
+            gather(0, false);
+            key(0, false);
+        }
+    }
+    __syncthreads();
+    const bool started = s_ab[1] == 0u;
+    uint32_t n = 0;
+    for (; started && n < nst; ++n) {
+        const uint32_t st = n & 1u;
+        // ---- region A(n): linked members, transition, stores ----
+        if (member) {
+            if (trace) trace[n * 8 + 0] = clock64();
+            if (n > 0) {
+                gather(n, true);
+                key(n, true);
+            }
+            if (trace) trace[n * 8 + 1] = clock64();
+            uint32_t v = (tid < cnt && ok) ? odd : 0u;
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+            if (lane == 0) warp_odd[tid >> 5] = v;
+            uint32_t upd = 0;
+            if (tid < cnt && ok) {
+                const uint32_t s = idx_of(st)[tid], o = out_of(st)[tid];
+                uint4 r[NV];
+#pragma unroll
+                for (uint32_t k = 0; k < NV; ++k) r[k] = rec_of(st)[pay_chunk<SB>(tid, k)];
+                const uint32_t y = tab[sel * a.tab_stride + r[0].x * 8u + o];
+                r[0].x = y;
+                r[0].y = r[0].y + 1u;
+                mix_acc<SB>(r, rk);
+#pragma unroll
+                for (uint32_t k = 0; k < NV; ++k) rec_of(st)[pay_chunk<SB>(tid, k)] = r[k];
+                uint4 e;
+                e.x = static_cast<uint32_t>(rk);
+                e.y = static_cast<uint32_t>(rk >> 32);
+                e.z = s;
+                e.w = y | (o << 16) | (sel << 24);
+                eff_of(st)[tid] = e;
+                if (a.state_log) {
+                    uint4 *lp = reinterpret_cast<uint4 *>(a.state_log + (static_cast<size_t>(n) * a.K + m0 + tid) * SB);
+#pragma unroll
+                    for (uint32_t k = 0; k < NV; ++k) __stcs(lp + k, r[k]);
+                }
+                upd = 1;
+            } else if (tid < cnt) {
+                s_rej = 1;  // a rejected member: this step's effects go out one by one
+            }
+            fence_proxy_async_smem();  // the staged effects are read by the bulk copy
+            const uint32_t umask = __ballot_sync(0xffffffffu, upd);
+            if (lane == 0) s_upd[tid >> 5] = umask;
+            __syncwarp();
+            const uint32_t c = lane % NV;
+#pragma unroll
+            for (uint32_t k = 0; k < NV; ++k) {
+                const uint32_t q = k * RPI + lane / NV;
+                if ((umask >> q) & 1u) {
+                    const uint32_t t = wbase + q;
+                    const uint32_t s = idx_of(st)[t];
+                    st_hint(reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(s) * SB) + c,
+                            rec_of(st)[pay_chunk<SB>(t, c)], keep_pol);
+                }
+            }
+            ok = 0;
+            if (trace) trace[n * 8 + 2] = clock64();
+        }
+        __syncthreads();  // region A done: stores issued, counts and effects staged
+        if (s_ab[0] != 0u) break;
+        // ---- region B(n): control thread publishes and waits; members run ahead ----
+        if (ctl) {
+            if (trace) trace[n * 8 + 0] = clock64();
+            uint32_t c = 0;
+            for (uint32_t w = 0; w < gs.members / 32u; ++w) c += warp_odd[w];
+            unsigned long long *word = &a.dev->slot[n % 3u];
+            if (blockIdx.x == 0) a.dev->slot[(n + 1u) % 3u] = 0ull;
+            const bool skip = (n == 0 && blockIdx.x == 1 && ld_volatile_u32(&a.dev->skip_arrival) != 0u);
+            if (!skip) red_release_add_u64(word, (1ull << 32) | c);
+            if (trace) trace[n * 8 + 1] = clock64();
+            if (a.effects && cnt > 0) {
+                if (s_rej == 0u) {
+                    bulk_store(reinterpret_cast<uint4 *>(a.effects) + static_cast<size_t>(n) * a.K + m0, eff_of(st),
+                               cnt * 16u);
+                } else {
+                    // error path: only the transitioned members' effects
+                    for (uint32_t t = 0; t < cnt; ++t)
+                        if ((s_upd[t >> 5] >> (t & 31u)) & 1u)
+                            reinterpret_cast<uint4 *>(a.effects)[static_cast<size_t>(n) * a.K + m0 + t] = eff_of(st)[t];
+                    s_rej = 0;
+                }
+                bulk_commit();
+                bulk_wait_read<1>();  // the staging buffer of step n - 1 is free again
+            }
+            if (cnt > 0 && n + 2u < nst) {
+                fence_proxy_async_smem();
+                issue(n + 2u);
+            }
+            if (trace) trace[n * 8 + 2] = clock64();
+            uint64_t t0 = 0;
+            unsigned long long w;
+            uint32_t spins = 0;
+            for (;;) {
+                w = ld_acquire_u64(word);
+                if ((w >> 32) >= G) break;
+                if ((++spins & 63u) == 0u) {
+                    if (ld_volatile_u32(&a.dev->abort) != 0u) {
+                        s_ab[1] = 1;
+                        break;
+                    }
+                    if (timed_out(t0, limit)) {
+                        latch_error(a.dev, DEV_E_TIMEOUT, n, blockIdx.x);
+                        atomicExch(&a.dev->abort, 1u);
+                        s_ab[1] = 1;
+                        break;
+                    }
+                }
+            }
+            const uint32_t d = (static_cast<uint32_t>(w & 0xffffffffull) > a.K / 2u) ? 1u : 0u;
+            s_sel = d;
+            if (blockIdx.x == 0 && a.decisions && s_ab[1] == 0u) a.decisions[n] = d;
+            if (trace) trace[n * 8 + 3] = clock64();
+        } else if (member && cnt > 0 && n + 1u < nst) {
+            if (!mbar_wait_bounded(&bar[(n + 1u) & 1u], ((n + 1u) >> 1) & 1u, limit)) {
+                latch_error(a.dev, DEV_E_TIMEOUT, n + 1u, blockIdx.x);
+                s_ab[1] = 1;
+            } else {
+                gather(n + 1u, false);
+                key(n + 1u, false);
+            }
+            if (trace) trace[n * 8 + 3] = clock64();
+        }
+        __syncthreads();  // region B done: decision of step n known, step n + 1 run ahead
+        if (s_ab[1] != 0u) break;
+        sel = s_sel;
+    }
+    cp_async_wait<0>();
+    if (ctl) {
+        bulk_wait_all<0>();
+        if (n < nst) {
+            // stopped early: wait (bounded) for the event copies still in flight
+            for (uint32_t j = n; j < issued; ++j) (void)mbar_wait_bounded(&bar[j & 1u], (j >> 1) & 1u, limit);
+        } else if (blockIdx.x == 0 && nst > 0) {
+            a.dev->sel = sel;
+            a.dev->step = nst;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
 // Persistent chain, split-phase (explicit session indices, K a multiple of 8,
 // at most 512 members per CTA; one CTA when K <= 512, else one CTA per SM).
 //
@@ -2392,6 +2736,99 @@ cudaError_t launch_chain_cta_link(const StepArgs &a, int SB, int P, size_t smem,
     if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
     void *args[] = {&map, &aa, &l, &shc};
     return cudaLaunchKernel(fn, dim3(1), dim3(member_threads + 32u), args, smem, s);
+}
+
+static const void *grid_link_fn(int SB, int P) {
+    return dispatch(SB, P, [](auto b, auto q) {
+        return reinterpret_cast<const void *>(&k_chain_grid_link<decltype(b)::value, decltype(q)::value>);
+    });
+}
+
+bool chain_grid_link_plan(int SB, int P, uint32_t K, uint64_t n_sessions, uint32_t n_sets, uint32_t tab_stride,
+                          int *grid, uint32_t *threads, size_t *smem, void *shape_out, size_t *scratch) {
+    if (K == 0 || K % 8u != 0u || n_sessions > 0xFFFFFFFFull || !encode_fn()) return false;
+    int dev = 0, sms = 0, max_optin = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return false;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return false;
+    if (cudaDeviceGetAttribute(&max_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+        return false;
+    GridLinkShape gs{};
+    TmaShape &sh = gs.t;
+    const uint32_t per = (K + static_cast<uint32_t>(sms) - 1u) / static_cast<uint32_t>(sms);
+    sh.chunk = (per + 7u) & ~7u;
+    const uint32_t g = (K + sh.chunk - 1u) / sh.chunk;
+    sh.n_boxes = (sh.chunk + 255u) / 256u;
+    sh.box_rows = (((sh.chunk + sh.n_boxes - 1u) / sh.n_boxes) + 7u) & ~7u;
+    sh.stage_pay = ((sh.n_boxes * sh.box_rows * static_cast<uint32_t>(P)) + 1023u) & ~1023u;
+    sh.stage_words = (sh.chunk + 3u) & ~3u;
+    gs.members = ((sh.chunk + 31u) / 32u) * 32u;
+    if (gs.members + 32u > 544u) return false;
+    const size_t bytes = 1024 + 2ull * sh.stage_pay + 6ull * sh.stage_words * 4 + ((2ull * tab_stride + 15u) & ~15ull) +
+                         2ull * sh.chunk * SB + 2ull * sh.chunk * 16 + 64;
+    if (bytes > static_cast<size_t>(max_optin)) return false;
+    const uint64_t words_per_set = (n_sessions + 31u) / 32u;
+    const size_t bits_bytes = (static_cast<size_t>(n_sets) * words_per_set * 4 + 255u) & ~static_cast<size_t>(255u);
+    const size_t need = bits_bytes + static_cast<size_t>(n_sets) * K * 4;
+    if (need > (1ull << 30)) return false;
+    const void *fn = grid_link_fn(SB, P);
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes)) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, static_cast<int>(gs.members + 32u), bytes) !=
+            cudaSuccess ||
+        per_sm < 1 || static_cast<long long>(per_sm) * sms < g)
+        return false;
+    *grid = static_cast<int>(g);
+    *threads = gs.members + 32u;
+    *smem = bytes;
+    *scratch = need;
+    static_assert(sizeof(GridLinkShape) <= 48, "shape buffer");
+    std::memcpy(shape_out, &gs, sizeof(gs));
+    return true;
+}
+
+cudaError_t launch_chain_grid_link(const StepArgs &a, int SB, int P, int grid, uint32_t threads, size_t smem,
+                                   const void *shape, void *scratch, cudaStream_t s) {
+    GridLinkShape gs;
+    std::memcpy(&gs, shape, sizeof(gs));
+    // [bitmaps, padded to 256 bytes][link words]: the link runs are read by
+    // 16-byte-aligned bulk copies
+    const uint64_t words_per_set = (a.n_sessions + 31u) / 32u;
+    const size_t bits_bytes = (static_cast<size_t>(a.n_sets) * words_per_set * 4 + 255u) & ~static_cast<size_t>(255u);
+    uint32_t *bits = static_cast<uint32_t *>(scratch);
+    uint32_t *lnk = reinterpret_cast<uint32_t *>(static_cast<uint8_t *>(scratch) + bits_bytes);
+    cudaError_t e = cudaMemsetAsync(bits, 0, static_cast<size_t>(a.n_sets) * words_per_set * 4, s);
+    if (e != cudaSuccess) return e;
+    int dev = 0, sms = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+    const size_t total = static_cast<size_t>(a.n_sets) * a.K;
+    const size_t want = (total + 255u) / 256u;
+    const unsigned blocks = static_cast<unsigned>(want < static_cast<size_t>(sms) * 8u ? want : static_cast<size_t>(sms) * 8u);
+    k_mark<<<blocks ? blocks : 1u, 256, 0, s>>>(a.idx, a.n_sets, a.K, a.n_sessions, words_per_set, bits);
+    k_flag<<<blocks ? blocks : 1u, 256, 0, s>>>(a.idx, a.n_sets, a.K, a.n_sessions, words_per_set, bits, lnk);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    const TmaShape &sh = gs.t;
+    EncodeTiled enc = encode_fn();
+    if (!enc) return cudaErrorNotSupported;
+    alignas(64) CUtensorMap map;
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(P), static_cast<cuuint64_t>(a.n_sets) * a.K};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(P)};
+    const cuuint32_t box[2] = {static_cast<cuuint32_t>(P), sh.box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUtensorMapSwizzle swz = P == 128 ? CU_TENSOR_MAP_SWIZZLE_128B
+                                   : P == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                             : CU_TENSOR_MAP_SWIZZLE_32B;
+    CUresult r = enc(&map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t *>(a.payload), dims, strides, box,
+                     estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    StepArgs aa = a;
+    const uint32_t *l = lnk;
+    void *args[] = {&map, &aa, &l, &gs};
+    return cudaLaunchCooperativeKernel(grid_link_fn(SB, P), dim3(grid), dim3(threads), args, smem, s);
 }
 
 static const void *split_fn(int SB, int P) {

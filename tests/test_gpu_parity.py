@@ -173,17 +173,20 @@ def test_launch_floor_probes_run(g, rc):
         rc.rc_free(ctx)
 
 
-@pytest.mark.parametrize("kernel", ["owned", "split", "tma", "plain"])
+@pytest.mark.parametrize("kernel", ["link", "owned", "split", "tma", "plain"])
 @pytest.mark.parametrize("SB,P", [(16, 32), (16, 64), (64, 128), (64, 32)])
 @pytest.mark.parametrize("K,N,identity", [(1032, 5000, False), (4104, 9001, False), (4104, 4200, False),
                                           (2048, 2048, True), (65536, 70000, False), (65536, 1 << 20, False)])
 def test_persistent_grid_kernels(g, rc, monkeypatch, kernel, SB, P, K, N, identity):
     """The cooperative persistent kernels: split-phase (explicit sessions, K a
     multiple of 8), TMA-fed and plain, on member counts that do not split
-    evenly over SMs, with sessions recurring from step to step (N near K)."""
+    evenly over SMs, with sessions recurring from step to step (N near K);
+    "link" is the grid chain split by links (the default for explicit
+    sessions), the others turn it off."""
     monkeypatch.setenv("RC_OWNED", "1" if kernel == "owned" else "0")
     monkeypatch.setenv("RC_SPLIT", "1" if kernel == "split" else "0")
     monkeypatch.setenv("RC_NO_TMA", "1" if kernel == "plain" else "0")
+    monkeypatch.setenv("RC_NO_GRID_LINK", "0" if kernel == "link" else "1")
     S = 256 if SB == 64 else 64
     tables, state0, outc, pay, idx = _inputs(50 + K % 11, K, S, SB, P, 3, N=None if identity else N)
     n = 5
@@ -192,12 +195,13 @@ def test_persistent_grid_kernels(g, rc, monkeypatch, kernel, SB, P, K, N, identi
     g.assert_same(got, want, f"grid {kernel} K={K} N={N} SB={SB} P={P}")
 
 
-@pytest.mark.parametrize("kernel", ["owned", "split", "tma", "plain"])
+@pytest.mark.parametrize("kernel", ["link", "owned", "split", "tma", "plain"])
 def test_grid_barrier_wait_is_bounded_every_grid_kernel(g, rc, monkeypatch, kernel):
     import torch
     monkeypatch.setenv("RC_OWNED", "1" if kernel == "owned" else "0")
     monkeypatch.setenv("RC_SPLIT", "1" if kernel == "split" else "0")
     monkeypatch.setenv("RC_NO_TMA", "1" if kernel == "plain" else "0")
+    monkeypatch.setenv("RC_NO_GRID_LINK", "0" if kernel == "link" else "1")
     K, S, SB, P, n = 8192, 16, 16, 64, 4
     tables, state0, outc, pay, idx = _inputs(19, K, S, SB, P, 2, N=9000)
     ctx = rc.rc_init(S, tables, SB, P, K, 9000, torch.cuda.current_stream())
