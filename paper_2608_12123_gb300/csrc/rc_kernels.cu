@@ -29,11 +29,27 @@ constexpr uint64_t kGamma = 0x9E3779B97F4A7C15ull;  // golden-ratio increment of
 constexpr uint64_t kFinA = 0xBF58476D1CE4E5B9ull;   // finaliser multipliers
 constexpr uint64_t kFinB = 0x94D049BB133111EBull;
 
+// z * c mod 2^64 from 32-bit parts: the wide product of the low words, plus
+// the two cross products (the high x high term vanishes mod 2^64) in the
+// high word.  Written out because the dependent chain is a little shorter
+// than the compiler's 64-bit multiply sequence (measured on GB300: 63.5 vs
+// 69 cycles a finaliser round with one warp, 79 vs 91 with two warps per SM
+// sub-partition); the result is the same.
+__device__ __forceinline__ uint64_t mul64c(uint64_t z, uint64_t c) {
+    const uint32_t zl = static_cast<uint32_t>(z), zh = static_cast<uint32_t>(z >> 32);
+    const uint32_t cl = static_cast<uint32_t>(c), ch = static_cast<uint32_t>(c >> 32);
+    uint64_t w;
+    asm("mul.wide.u32 %0, %1, %2;" : "=l"(w) : "r"(zl), "r"(cl));
+    uint32_t cross;
+    asm("mad.lo.u32 %0, %1, %2, %3;" : "=r"(cross) : "r"(zl), "r"(ch), "r"(zh * cl));
+    return w + (static_cast<uint64_t>(cross) << 32);
+}
+
 __device__ __forceinline__ uint64_t fin64(uint64_t z) {
     z ^= z >> 30;
-    z *= kFinA;
+    z = mul64c(z, kFinA);
     z ^= z >> 27;
-    z *= kFinB;
+    z = mul64c(z, kFinB);
     return z ^ (z >> 31);
 }
 
@@ -81,7 +97,7 @@ __device__ __forceinline__ void rec_set_word(uint4 (&r)[NV], uint64_t v) {
 
 template <int J, int NV>
 __device__ __forceinline__ void mix_acc_word(uint4 (&r)[NV], uint64_t rk) {
-    rec_set_word<1 + J, NV>(r, (rec_word<1 + J, NV>(r) ^ rotl64c<8 * J>(rk)) * kGamma);
+    rec_set_word<1 + J, NV>(r, mul64c(rec_word<1 + J, NV>(r) ^ rotl64c<8 * J>(rk), kGamma));
 }
 
 // acc update: one word for the 16-byte record, seven rotated words for 64.
