@@ -381,23 +381,26 @@ int run_cond(rc_ctx *c, const rc::StepArgs &a) {
 
 // ---- device resident: persistent kernel ------------------------------------
 int run_persist(rc_ctx *c, const rc::StepArgs &a) {
-    if (a.idx && c->use_owned && c->coop) {
+    if (a.idx && c->use_owned && c->coop && static_cast<uint64_t>(a.n_sets) * a.K < (1ull << 31) - 1024u) {
         int grid = 0;
         uint32_t threads = 0;
         size_t smem = 0;
         alignas(8) unsigned char shape[32];
         if (rc::chain_owned_plan(c->SB, c->P, a.K, c->n_sessions, c->tab_stride, &grid, &threads, &smem, shape)) {
             const size_t nev = static_cast<size_t>(a.n_sets) * a.K;
-            int rc = ensure(c, c->route_buf, nev * 12 + static_cast<size_t>(a.n_sets) * (grid + 1) * 4 + 64);
+            const size_t words = (nev * 12 + static_cast<size_t>(a.n_sets) * (grid + 1) * 4 + 255u) & ~size_t(255);
+            int rc = ensure(c, c->route_buf, words + nev * c->P);
             if (rc != RC_OK) return rc;
             uint32_t *pm = static_cast<uint32_t *>(c->route_buf.p);
             uint32_t *ps = pm + nev, *po = ps + nev, *off = po + nev;
+            uint8_t *pay_routed = static_cast<uint8_t *>(c->route_buf.p) + words;
             RC_CUDA(c, cudaMemsetAsync(c->dev->slot4, 0, sizeof(c->dev->slot4), c->stream));
             RC_CUDA(c, cudaMemsetAsync(&c->dev->abort, 0, sizeof(uint32_t), c->stream));
-            c->last_launches = 2;  // routing pass + chain
+            c->last_launches = 3;  // routing pass, payload in routed order, chain
             RC_CUDA(c, rc::launch_route(a, shape, pm, ps, po, off, c->stream));
+            RC_CUDA(c, rc::launch_permute_payload(a, c->P, shape, pm, off, pay_routed, c->stream));
             RC_CUDA(c, rc::launch_chain_owned(a, c->SB, c->P, grid, threads, smem, shape, pm, ps, po, off,
-                                              c->stream));
+                                              pay_routed, c->stream));
             RC_CUDA(c, cudaMemsetAsync(&c->dev->skip_arrival, 0, sizeof(uint32_t), c->stream));
             return RC_OK;
         }

@@ -129,9 +129,15 @@ bool chain_owned_plan(int state_bytes, int payload_bytes, uint32_t K, uint64_t n
                       int *grid, uint32_t *threads, size_t *smem, void *shape_out);
 cudaError_t launch_route(const StepArgs &a, const void *shape, uint32_t *perm_m, uint32_t *perm_s, uint32_t *perm_o,
                          uint32_t *off, cudaStream_t s);
+// launch_permute_payload writes each cohort's payload rows in routed order
+// (n_sets * K * payload_bytes bytes at pay_routed), which the chain then
+// loads as tensor tiles.
+cudaError_t launch_permute_payload(const StepArgs &a, int payload_bytes, const void *shape, const uint32_t *perm_m,
+                                   const uint32_t *off, uint8_t *pay_routed, cudaStream_t s);
 cudaError_t launch_chain_owned(const StepArgs &a, int state_bytes, int payload_bytes, int grid, uint32_t threads,
                                size_t smem, const void *shape, const uint32_t *perm_m, const uint32_t *perm_s,
-                               const uint32_t *perm_o, const uint32_t *off, cudaStream_t s);
+                               const uint32_t *perm_o, const uint32_t *off, const uint8_t *pay_routed,
+                               cudaStream_t s);
 
 // Writes decisions[0..n) = 0 and sel = 0 (an empty cohort decides 0).
 cudaError_t launch_empty_cohorts(const StepArgs &a, cudaStream_t s);

@@ -2071,6 +2071,27 @@ __global__ void k_route(const uint32_t *idx, const uint32_t *outcome, uint32_t n
     }
 }
 
+// Copies each cohort's payload rows into routed order: row i of cohort j
+// becomes the payload of member perm_m[j][i], so that every CTA's run of a
+// cohort is a block of consecutive rows that tensor tiles can load.  Rows
+// past the cohort's routed count (invalid sessions) are left alone.
+__global__ void k_permute_payload(const uint8_t *payload, const uint32_t *perm_m, const uint32_t *off,
+                                  uint32_t n_sets, uint32_t K, uint32_t G, uint32_t P, uint8_t *out) {
+    const uint32_t nc = P / 16u;
+    const size_t total = static_cast<size_t>(n_sets) * K * nc;
+    for (size_t q = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; q < total;
+         q += static_cast<size_t>(gridDim.x) * blockDim.x) {
+        const size_t e = q / nc;
+        const uint32_t c = static_cast<uint32_t>(q % nc);
+        const size_t j = e / K;
+        const uint32_t i = static_cast<uint32_t>(e % K);
+        if (i >= off[j * (G + 1u) + G]) continue;
+        const uint32_t m = perm_m[e];
+        reinterpret_cast<uint4 *>(out)[e * nc + c] =
+            __ldg(reinterpret_cast<const uint4 *>(payload + (j * K + m) * P) + c);
+    }
+}
+
 struct OwnedShape {
     uint32_t G;    // CTAs
     uint32_t per;  // sessions owned per CTA
@@ -2093,11 +2114,13 @@ struct Routed {
 
 template <int SB, int P, bool RES>
 __global__ void __launch_bounds__(512, 1)
-    k_chain_owned(StepArgs a, OwnedShape sh, const uint32_t *perm_m, const uint32_t *perm_s,
-                  const uint32_t *perm_o, const uint32_t *off) {
+    k_chain_owned(const __grid_constant__ CUtensorMap tmap, StepArgs a, OwnedShape sh, const uint32_t *perm_m,
+                  const uint32_t *perm_s, const uint32_t *perm_o, const uint32_t *off) {
     constexpr int NV = SB / 16;
     constexpr uint32_t NC = P / 16;
+    constexpr uint32_t kTileRows = 256;
     extern __shared__ __align__(16) uint8_t dsm[];
+    __shared__ __align__(8) uint64_t tbar[2];
     __shared__ uint32_t warp_odd[16];
     __shared__ uint32_t s_sel, s_abort;
     const uint32_t tid = threadIdx.x;
@@ -2113,12 +2136,16 @@ __global__ void __launch_bounds__(512, 1)
     long long *trace = (a.trace && tid == 0 && (b == 0 || b == G - 1))
                            ? a.trace + (b == 0 ? 0 : static_cast<size_t>(nst) * 8)
                            : nullptr;
-    // shared layout: [tables][payload rows: 2 stages x T][record stage: T (not RES)][owned states or records]
-    uint8_t *tab = dsm;
-    uint4 *pay = reinterpret_cast<uint4 *>(dsm + 2 * a.tab_stride);
-    uint4 *rec_st = pay + 2ull * T * NC;
-    uint8_t *owned = reinterpret_cast<uint8_t *>(rec_st + (RES ? 0ull : static_cast<size_t>(T) * NV));
+    // shared layout: [payload tiles: 2 stages x 2 tiles of 256 rows, 1024-aligned][tables]
+    // [record stage: T (not RES)][owned states (u16) or records]
+    const uint32_t raw = smem_addr(dsm);
+    uint8_t *const pay = dsm + (((raw + 1023u) & ~1023u) - raw);
+    constexpr uint32_t kStage = 2u * kTileRows * P;
+    uint8_t *tab = pay + 2u * kStage;
+    uint4 *rec_st = reinterpret_cast<uint4 *>(tab + 2 * a.tab_stride);
+    uint16_t *owned = reinterpret_cast<uint16_t *>(rec_st + (RES ? 0ull : static_cast<size_t>(T) * NV));
     uint4 *owned_rec = reinterpret_cast<uint4 *>(owned);  // RES: [per][NV]
+    const uint64_t stream_pol = policy_evict_first();
 
     stage_tables(tab, a.tables, a.tab_stride, 2, 0);
     for (uint32_t ls = tid; ls < own; ls += T) {
@@ -2127,12 +2154,16 @@ __global__ void __launch_bounds__(512, 1)
 #pragma unroll
             for (int k = 0; k < NV; ++k) owned_rec[static_cast<size_t>(ls) * NV + k] = rp[k];
         } else {
-            owned[ls] = static_cast<uint8_t>(__ldg(reinterpret_cast<const uint32_t *>(rp)));
+            const uint32_t x0 = __ldg(reinterpret_cast<const uint32_t *>(rp));
+            owned[ls] = static_cast<uint16_t>(x0 < a.S ? x0 : 0xFFFFu);  // >= S stays >= S
         }
     }
     if (tid == 0) {
         s_sel = ld_volatile_u32(&a.dev->sel) & 1u;
         s_abort = 0;
+        mbar_init(&tbar[0], 1);
+        mbar_init(&tbar[1], 1);
+        fence_mbar_init();
     }
 
     // run of step j for this CTA (two plain loads; clamped so that no branch waits on them)
@@ -2154,23 +2185,22 @@ __global__ void __launch_bounds__(512, 1)
         r.o = __ldg(perm_o + e);
         r.valid = v ? 1u : 0u;
     };
-    // The warp's rows and records are copied warp-cooperatively: NC (NV) lanes
-    // take the 16-byte chunks of one payload row (record), so one copy
-    // instruction of the warp touches 32 / NC whole rows instead of a chunk of
-    // 32 rows; each lane learns the row's member or session by a shuffle.
+    // The run of step j sits in rows [j*K + lo, j*K + hi) of the routed
+    // payload copy: thread 0 loads it as one or two 256-row tensor tiles
+    // (rows past the run are loaded and ignored).  Records are gathered
+    // warp-cooperatively: NV lanes take the 16-byte chunks of one record.
     const uint32_t lane = tid & 31u, wbase = tid & ~31u;
-    auto stage_row = [&](uint32_t j, const Routed &r) {  // all lanes of the warp
-        constexpr uint32_t RPI = 32u / NC;
-        uint4 *dst = pay + static_cast<size_t>(j & 1u) * T * NC;
-        const size_t set0 = static_cast<size_t>(j % a.n_sets) * a.K;
-        const uint32_t c = lane % NC;
-#pragma unroll
-        for (uint32_t k = 0; k < NC; ++k) {
-            const uint32_t from = k * RPI + lane / NC;
-            const uint32_t m = __shfl_sync(0xffffffffu, r.m, from);
-            const uint32_t v = __shfl_sync(0xffffffffu, r.valid, from);
-            if (v) cp_async16(dst + pay_chunk<P>(wbase + from, c), reinterpret_cast<const uint4 *>(a.payload + (set0 + m) * P) + c);
-        }
+    uint32_t tiles_issued = 0;  // thread 0: steps [0, tiles_issued) have had their tiles issued
+    auto stage_tiles = [&](uint32_t j, uint32_t lo, uint32_t hi) {  // thread 0
+        if (j >= nst) return;
+        tiles_issued = j + 1u;
+        const uint32_t nb = (hi - lo) > kTileRows ? 2u : 1u;
+        uint64_t *bb = &tbar[j & 1u];
+        mbar_arrive_expect_tx(bb, nb * kTileRows * P);
+        const int32_t row0 = static_cast<int32_t>((j % a.n_sets) * a.K + lo);
+        for (uint32_t q = 0; q < nb; ++q)
+            tma_load_2d_hint(pay + (j & 1u) * kStage + q * kTileRows * P, &tmap, 0,
+                             row0 + static_cast<int32_t>(q * kTileRows), bb, stream_pol);
     };
     auto stage_record = [&](const Routed &r) {  // all lanes of the warp
         if constexpr (!RES) {
@@ -2220,9 +2250,8 @@ __global__ void __launch_bounds__(512, 1)
     load_run(2, lo2, hi2);
     load_entry(0, lo0, hi0, r0);
     load_entry(1, lo1, hi1, r1);
-    stage_row(0, r0);
-    cp_async_commit();
-    __syncthreads();
+    __syncthreads();  // mbarriers initialised
+    if (tid == 0) stage_tiles(0, lo0, hi0);
     uint32_t sel = s_sel;
     uint32_t low_prev[4] = {0u, 0u, 0u, 0u};
 
@@ -2232,10 +2261,15 @@ __global__ void __launch_bounds__(512, 1)
         load_entry(n + 2u, lo2, hi2, r2);
         stage_record(r0);           // records of step n (the previous step's writes are done)
         cp_async_commit();
-        stage_row(n + 1u, r1);      // rows of step n + 1
-        cp_async_commit();
-        cp_async_wait<2>();         // this lane's row copies of step n are here
-        __syncwarp();               // and so are the other lanes' (the warp's rows)
+        if (tid == 0) {             // tiles of step n + 1 into the stage step n - 1 used
+            fence_proxy_async_smem();
+            stage_tiles(n + 1u, lo1, (n + 1u < nst) ? hi1 : lo1);
+        }
+        if (!mbar_wait_bounded(&tbar[n & 1u], (n >> 1) & 1u, limit)) {  // tiles of step n
+            latch_error(a.dev, DEV_E_TIMEOUT, n, b);
+            atomicExch(&a.dev->abort, 1u);
+            s_abort = 1;
+        }
         if (trace) trace[n * 8 + 1] = clock64();
         const size_t e0 = static_cast<size_t>(n % a.n_sets) * a.K;
         const uint32_t cnt0 = hi0 - lo0;
@@ -2248,10 +2282,8 @@ __global__ void __launch_bounds__(512, 1)
             if (x >= a.S || r0.o >= 8u) {
                 latch_error(a.dev, DEV_E_STATE, n, r0.m);
             } else {
-                const uint4 *stage = pay + static_cast<size_t>(n & 1u) * T * NC;
                 uint4 pw[NC];
-#pragma unroll
-                for (uint32_t k = 0; k < NC; ++k) pw[k] = stage[pay_chunk<P>(tid, k)];
+                read_payload_swizzled<P>(pw, pay + (n & 1u) * kStage, tid);
                 rk = route_key<P>(x, r0.o, pw);
                 odd = static_cast<uint32_t>(rk & 1u);
                 ok = true;
@@ -2295,7 +2327,7 @@ __global__ void __launch_bounds__(512, 1)
         __syncthreads();
         if (s_abort) break;
         if (n > 0) sel = s_sel;
-        cp_async_wait<1>();  // the warp's records of step n are here
+        cp_async_wait<0>();  // the warp's records of step n are here
         __syncwarp();
         if (trace) trace[n * 8 + 6] = clock64();
         // --- next state, record and effect (body chosen by the decision of step n - 1) ---
@@ -2312,7 +2344,7 @@ __global__ void __launch_bounds__(512, 1)
 #pragma unroll
                 for (int k = 0; k < NV; ++k) owned_rec[static_cast<size_t>(ls) * NV + k] = rr[k];
             } else {
-                owned[ls] = static_cast<uint8_t>(y);
+                owned[ls] = static_cast<uint16_t>(y);
                 if (coop) {
 #pragma unroll
                     for (int k = 0; k < NV; ++k) rec_st[static_cast<size_t>(tid) * NV + k] = rr[k];
@@ -2397,6 +2429,10 @@ __global__ void __launch_bounds__(512, 1)
         hi2 = hi3;
     }
     cp_async_wait<0>();
+    if (tid == 0) {  // the tiles still in flight after an early stop (bounded)
+        for (uint32_t j = tiles_issued >= 2u ? tiles_issued - 2u : 0u; j < tiles_issued; ++j)
+            (void)mbar_wait_bounded(&tbar[j & 1u], (j >> 1) & 1u, limit);
+    }
     if (tid == 0 && !s_abort && nst > 0) {
         s_sel = wait_count(nst - 1u, low_prev);
         if (b == 0 && !s_abort) {
@@ -2929,7 +2965,7 @@ static const void *owned_fn(int SB, int P, bool res) {
 
 bool chain_owned_plan(int SB, int P, uint32_t K, uint64_t N, uint32_t tab_stride, int *grid, uint32_t *threads,
                       size_t *smem, void *shape_out) {
-    if (K == 0) return false;
+    if (K == 0 || !encode_fn()) return false;
     int dev = 0, sms = 0, max_optin = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return false;
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return false;
@@ -2944,9 +2980,10 @@ bool chain_owned_plan(int SB, int P, uint32_t K, uint64_t N, uint32_t tab_stride
     uint32_t thr = ((want + want / 4u + 31u) / 32u) * 32u;
     if (thr < 32u) thr = 32u;
     if (thr > 512u) thr = 512u;
-    const size_t base = 2 * static_cast<size_t>(tab_stride) + 2ull * thr * P;
+    // [1024-aligned payload tiles: 2 stages x 2 x 256 rows][tables][record stage][owned states]
+    const size_t base = 1024 + 4ull * 256 * P + 2 * static_cast<size_t>(tab_stride);
     const size_t res_bytes = base + static_cast<size_t>(sh.per) * SB;
-    const size_t x_bytes = base + static_cast<size_t>(thr) * SB + ((static_cast<size_t>(sh.per) + 15u) & ~size_t(15));
+    const size_t x_bytes = base + static_cast<size_t>(thr) * SB + ((static_cast<size_t>(sh.per) * 2 + 15u) & ~size_t(15));
     sh.res = res_bytes + 2048 <= static_cast<size_t>(max_optin) ? 1u : 0u;
     const size_t bytes = sh.res ? res_bytes : x_bytes;
     if (bytes + 2048 > static_cast<size_t>(max_optin)) return false;
@@ -2976,13 +3013,40 @@ cudaError_t launch_route(const StepArgs &a, const void *shape, uint32_t *perm_m,
     return cudaGetLastError();
 }
 
+cudaError_t launch_permute_payload(const StepArgs &a, int P, const void *shape, const uint32_t *perm_m,
+                                   const uint32_t *off, uint8_t *pay_routed, cudaStream_t s) {
+    const OwnedShape &sh = *static_cast<const OwnedShape *>(shape);
+    int dev = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+    k_permute_payload<<<static_cast<unsigned>(sms) * 8u, 256, 0, s>>>(a.payload, perm_m, off, a.n_sets, a.K, sh.G,
+                                                                      static_cast<uint32_t>(P), pay_routed);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_chain_owned(const StepArgs &a, int SB, int P, int grid, uint32_t threads, size_t smem,
                                const void *shape, const uint32_t *perm_m, const uint32_t *perm_s,
-                               const uint32_t *perm_o, const uint32_t *off, cudaStream_t s) {
+                               const uint32_t *perm_o, const uint32_t *off, const uint8_t *pay_routed,
+                               cudaStream_t s) {
     const OwnedShape &sh = *static_cast<const OwnedShape *>(shape);
+    EncodeTiled enc = encode_fn();
+    if (!enc) return cudaErrorNotSupported;
+    alignas(64) CUtensorMap map;
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(P), static_cast<cuuint64_t>(a.n_sets) * a.K};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(P)};
+    const cuuint32_t box[2] = {static_cast<cuuint32_t>(P), 256u};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUtensorMapSwizzle swz = P == 128 ? CU_TENSOR_MAP_SWIZZLE_128B
+                                   : P == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                             : CU_TENSOR_MAP_SWIZZLE_32B;
+    CUresult r = enc(&map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t *>(pay_routed), dims, strides, box,
+                     estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
     StepArgs aa = a;
     OwnedShape shc = sh;
-    void *args[] = {&aa, &shc, &perm_m, &perm_s, &perm_o, &off};
+    void *args[] = {&map, &aa, &shc, &perm_m, &perm_s, &perm_o, &off};
     return cudaLaunchCooperativeKernel(owned_fn(SB, P, sh.res != 0), dim3(grid), dim3(threads), args, smem, s);
 }
 
