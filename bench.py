@@ -255,6 +255,12 @@ def native(args):
     if not args.large_k_only:
         w = make_config2()
         nc = w["n_cohorts"]
+        # how much of the replay a resident cohort path can reach (Section 4):
+        # F, P*, U from the library's host code, A from its former
+        t_op = time.perf_counter()
+        opp = rc.opportunity_shares(w["arr"].t_ns, w["arr"].route, w["panel"].n_labels, K, C2["delta_ns"],
+                                    w["members"].size)
+        opp_s = time.perf_counter() - t_op
         S, SB, P = C2["S"], C2["state_bytes"], C2["payload_bytes"]
         ctx = rc.rc_init(S, w["tables"], SB, P, K, w["arr"].n_sessions, stream)
         state = torch.from_numpy(w["state0"].copy()).cuda()
@@ -350,6 +356,12 @@ def native(args):
                        "events": w["arr"].n, "mechanism": "resident_persist (one persistent CTA)",
                        "l2": "flushed between timed steps (512 MiB write)",
                        "parallelism": "replicas" if world > 1 else "single GPU"},
+            "opportunity": {"F": round(opp["F"], 6), "P_star": round(opp["P"], 6), "U": round(opp["U"], 6),
+                            "A": round(opp["A"], 6),
+                            "G": None if opp["G"] is None else round(opp["G"], 6),
+                            "R_A": None if opp["R_A"] is None else round(opp["R_A"], 6),
+                            "events": opp["n"], "counts": opp["counts"], "host_s": round(opp_s, 3),
+                            "by": "rc_opportunity (F Eq. 2, P* Eq. 6 / Algorithm 1, U Eqs. 3-4) and the former (A)"},
             "host_rt_us_per_invocation": round(mech_us["host_rt"] / world, 4),
             "ratio_host_rt_over_resident": round(mech_us["host_rt"] / mech_us["resident_persist"], 3),
             "mechanisms_us_per_invocation": {k: round(v, 4) for k, v in mech_us.items()},

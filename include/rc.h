@@ -255,6 +255,25 @@ int64_t rc_former_pop_many(rc_former *f, uint64_t max_cohorts, int64_t *members_
 int rc_former_counts(rc_former *f, int64_t *pushed, int64_t *launched, int64_t *fallback);
 int rc_former_free(rc_former *f);
 
+/* Opportunity counts of an event set (host, Section 4), at threshold K and
+ * deadline delta_ns for every route:
+ *   fixed  events in (route, window) buckets holding >= K events, windows
+ *          [origin_ns + w delta, origin_ns + (w + 1) delta) (Eq. 2, F);
+ *   exact  the most events that batches of >= K same-route events, each
+ *          spanning at most delta, can hold (Eq. 6, P*; computed by the
+ *          deque recurrence of Algorithm 1);
+ *   upper  events i for which some release tau in [t_i, t_i + delta] sees
+ *          >= K same-route events in [tau - delta, tau] (Eqs. 3-4, U).
+ * Shares are these counts over n; with the former's launched count A,
+ * G = (P* - F) / (U - F) (Eq. 7) and R_A = (A - F) / (P* - F) (Eq. 9).
+ * Inputs are host arrays of n events in any order; route < n_routes.
+ * Returns RC_E_INVAL on K == 0, delta_ns <= 0 or a route out of range.   */
+typedef struct {
+    uint64_t n, fixed, exact, upper;
+} rc_opportunity_counts;
+int rc_opportunity(const int64_t *t_ns, const uint32_t *route, uint64_t n, uint32_t n_routes, uint32_t K,
+                   int64_t delta_ns, int64_t origin_ns, rc_opportunity_counts *out);
+
 #ifdef __cplusplus
 }
 #endif

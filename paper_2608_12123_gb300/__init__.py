@@ -44,7 +44,11 @@ MECHANISMS = {"host_rt": RC_MECH_HOST_RT, "resident_cond": RC_MECH_RESIDENT_COND
 EXPORTS = ("rc_init", "rc_cohort_step", "rc_chain", "rc_free", "rc_last_error", "rc_sync",
            "rc_get_decision", "rc_set_decision", "rc_set_wait_limits", "rc_launch_floor",
            "rc_debug_skip_arrival", "rc_last_chain_stats", "rc_set_trace", "rc_cohort_step_noalloc", "rc_former_create", "rc_former_push", "rc_former_pop",
-           "rc_former_push_many", "rc_former_pop_many", "rc_former_counts", "rc_former_free")
+           "rc_former_push_many", "rc_former_pop_many", "rc_former_counts", "rc_former_free", "rc_opportunity")
+
+
+class rc_opportunity_counts(C.Structure):
+    _fields_ = [("n", C.c_uint64), ("fixed", C.c_uint64), ("exact", C.c_uint64), ("upper", C.c_uint64)]
 
 
 class rc_events(C.Structure):
@@ -81,6 +85,7 @@ def _load():
         "rc_former_pop_many": (i64, [vp, u64, vp, vp, vp]),
         "rc_former_counts": (i, [vp, P(i64), P(i64), P(i64)]),
         "rc_former_free": (i, [vp]),
+        "rc_opportunity": (i, [vp, vp, u64, u32, u32, i64, i64, P(rc_opportunity_counts)]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -312,3 +317,30 @@ def form_cohorts(t_ns, route, session, n_routes, K, delta_ns):
         return members[:nc], tau[:nc], rr[:nc]
     finally:
         rc_former_free(f)
+
+
+def rc_opportunity(t_ns, route, n_routes, K, delta_ns, origin_ns=0):
+    """Counts {n, fixed, exact, upper}: the events that fixed windows (F, Eq. 2),
+    the exact offline packing (P*, Eq. 6) and the upper bound (U, Eqs. 3-4)
+    serve at threshold K and deadline delta_ns."""
+    import numpy as np
+    t_ns = np.ascontiguousarray(t_ns, dtype=np.int64)
+    route = np.ascontiguousarray(route, dtype=np.uint32)
+    out = rc_opportunity_counts()
+    rc = _lib.rc_opportunity(t_ns.ctypes.data, route.ctypes.data, len(t_ns), n_routes, K, delta_ns, origin_ns,
+                             C.byref(out))
+    if rc != RC_OK:
+        raise RcError(rc, "rc_opportunity rejected its arguments")
+    return dict(n=int(out.n), fixed=int(out.fixed), exact=int(out.exact), upper=int(out.upper))
+
+
+def opportunity_shares(t_ns, route, n_routes, K, delta_ns, launched, origin_ns=0):
+    """F, P*, U and A as fractions of the events, G (Eq. 7) and R_A (Eq. 9)
+    from rc_opportunity and the former's launched-event count."""
+    c = rc_opportunity(t_ns, route, n_routes, K, delta_ns, origin_ns)
+    n, f, p, u = c["n"], c["fixed"], c["exact"], c["upper"]
+    out = dict(n=n, F=f / n if n else 0.0, P=p / n if n else 0.0, U=u / n if n else 0.0,
+               A=launched / n if n else 0.0, counts=dict(F=f, P=p, U=u, A=int(launched)))
+    out["G"] = (p - f) / (u - f) if u > f else None
+    out["R_A"] = (launched - f) / (p - f) if p > f else None
+    return out

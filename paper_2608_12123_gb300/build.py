@@ -22,7 +22,7 @@ ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++20", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC,
               "--expt-relaxed-constexpr"]
 CU_SOURCES = ["rc_kernels.cu", "rc_api.cu"]
-CXX_SOURCES = ["rc_former.cpp"]
+CXX_SOURCES = ["rc_former.cpp", "rc_opportunity.cpp"]
 
 
 def _nvcc() -> str:
