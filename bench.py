@@ -61,6 +61,8 @@ def parse_args():
     p.add_argument("--only-resident", action="store_true",
                    help="time only the resident chain of the headline workload (profiling)")
     p.add_argument("--no-flush", action="store_true", help="do not allocate or write the L2 flush buffer (profiling)")
+    p.add_argument("--sweep", action="store_true",
+                   help="instead of the bench line: horizon sweep H x N x mechanism and the safe suffix K_r")
     return p.parse_args()
 
 
@@ -525,8 +527,83 @@ def reference(args):
             "e2e": {"value": round(us, 4), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
+def sweep(args):
+    """The paper's horizon grid (H in {2, 8, 32} steps per call x N in {256,
+    2048, 16384} members per step x mechanism; Sections 7.3 and 8.1) and the
+    safe suffix K_r (the smallest K from which the resident GPU step beats the
+    CPU oracle at every tested size, Section 3).  Inputs: cohorts of N
+    distinct sessions out of 4N, 64-byte payloads, 16-byte state, S = 64, a
+    ring of 64 cohorts."""
+    import torch
+    import paper_2608_12123_gb300 as rc
+    import oracle
+    stream = torch.cuda.current_stream()
+    S, SB, P, ring = 64, 16, 64, 64
+    tables = wl.make_tables(S, wl.stream_seed(20, wl.Purpose.TABLE))
+    mechs = {"resident_persist": rc.RC_MECH_RESIDENT_PERSIST, "resident_cond": rc.RC_MECH_RESIDENT_COND,
+             "host_rt": rc.RC_MECH_HOST_RT, "fixed_nested": rc.RC_MECH_FIXED_NESTED}
+
+    def setup(N):
+        outc, pay, idx = wl.make_cohort_events(20, ring, N, P, n_sessions=4 * N)
+        state0 = wl.make_state(4 * N, S, SB, wl.stream_seed(20, wl.Purpose.STATE, N))
+        ctx = rc.rc_init(S, tables, SB, P, N, 4 * N, stream)
+        dev_ev = (torch.from_numpy(outc.view(np.int32)).cuda(), torch.from_numpy(pay).cuda(),
+                  torch.from_numpy(idx.view(np.int32)).cuda())
+        state = torch.from_numpy(state0.copy()).cuda()
+        dec = torch.zeros(ring, dtype=torch.int32, device="cuda")
+        return ctx, dev_ev, state, dec, (outc, pay, idx, state0)
+
+    horizon = {}
+    for N in (256, 2048, 16384):
+        ctx, dev_ev, state, dec, _ = setup(N)
+        reps = 40 if N < 16384 else 15
+        horizon[str(N)] = {}
+        for name, mech in mechs.items():
+            horizon[str(N)][name] = {}
+            for Hh in (2, 8, 32):
+                t = []
+                for r in range(reps + 3):
+                    ms, _ = chain_on_window(rc, ctx, mech, state, dev_ev, (r * Hh) % (ring - Hh), Hh, N, dec, None)
+                    if r >= 3:
+                        t.append(ms * 1000.0)
+                horizon[str(N)][name][str(Hh)] = round(float(np.median(t)), 2)
+        rc.rc_free(ctx)
+    ratio = {N: {Hh: round(horizon[N]["host_rt"][Hh] / horizon[N]["resident_persist"][Hh], 3) for Hh in ("2", "8", "32")}
+             for N in horizon}
+
+    per_k = {}
+    for K in (32, 64, 128, 256, 512, 1024, 2048, 4096, 16384, 65536):
+        ctx, dev_ev, state, dec, (outc, pay, idx, state0) = setup(K)
+        t = []
+        for r in range(6):
+            ms, _ = chain_on_window(rc, ctx, rc.RC_MECH_RESIDENT_PERSIST, state, dev_ev, 0, ring, K, dec, None)
+            if r >= 1:
+                t.append(ms * 1000.0 / ring)
+        rc.rc_free(ctx)
+        m = 16  # oracle steps, single thread, as it stands
+        st = state0.copy()
+        t0 = time.perf_counter()
+        oracle.chain(tables, st, outc[:m], pay[:m], idx[:m], m, log=False)
+        cpu = (time.perf_counter() - t0) * 1e6 / m
+        per_k[str(K)] = {"gpu_resident_us": round(float(np.median(t)), 4), "cpu_oracle_us": round(cpu, 2)}
+    ks = sorted(int(k) for k in per_k)
+    k_r = None
+    for i, k in enumerate(ks):
+        if all(per_k[str(k2)]["gpu_resident_us"] < per_k[str(k2)]["cpu_oracle_us"] for k2 in ks[i:]):
+            k_r = k
+            break
+    return {"sweep": {"workload": "cohorts of N distinct sessions out of 4N, 16-byte state, 64-byte payload, "
+                                  "S=64, ring of 64 cohorts; medians of repeated calls",
+                      "horizon_us_per_call": horizon, "ratio_host_rt_over_resident": ratio,
+                      "safe_suffix": {"per_K_us_per_invocation": per_k, "K_r": k_r,
+                                      "cpu": "oracle chain, one thread, 16 steps per K"}}}
+
+
 def main():
     args = parse_args()
+    if args.sweep:
+        print(json.dumps(sweep(args)))
+        return
     out = reference(args) if args.impl == "reference" else native(args)
     if out is not None:
         print(json.dumps(out))
