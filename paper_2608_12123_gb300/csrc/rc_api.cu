@@ -92,6 +92,7 @@ struct rc_ctx {
     bool no_link = false;   // RC_NO_LINK=1 turns off the linked single-CTA kernels
     bool no_prod = false;   // RC_NO_PROD=1 keeps the linked kernel without a producer warp
     bool no_grid_link = false;  // RC_NO_GRID_LINK=1 turns off the grid chain split by links
+    bool no_cluster = false;    // RC_NO_CLUSTER=1 turns off the cluster chain (512 < K <= 8192)
     bool use_split = false;  // RC_SPLIT=1 selects the split-phase chain (slower on GB300 so far)
     bool use_owned = false;  // RC_OWNED=1 selects the session-owned chain
     Buf route_buf;           // session-owned chain: routed member lists
@@ -445,6 +446,13 @@ int run_persist(rc_ctx *c, const rc::StepArgs &a) {
             return RC_OK;
         }
     }
+    if (!c->no_cluster) {
+        uint32_t cluster = 0, threads = 0;
+        if (rc::chain_cluster_plan(c->SB, c->P, a.K, &cluster, &threads)) {
+            RC_CUDA(c, rc::launch_chain_cluster(a, c->SB, c->P, cluster, threads, c->stream));
+            return RC_OK;
+        }
+    }
     if (!c->coop) return fail(c, RC_E_UNSUPPORTED, "device lacks cooperative launch");
     RC_CUDA(c, cudaMemsetAsync(c->dev->slot, 0, sizeof(c->dev->slot), c->stream));
     RC_CUDA(c, cudaMemsetAsync(&c->dev->abort, 0, sizeof(uint32_t), c->stream));
@@ -598,6 +606,8 @@ int rc_init(rc_ctx **out, uint32_t S, const uint8_t *table, uint32_t state_bytes
         c->no_prod = q && q[0] == '1';
         const char *gl = std::getenv("RC_NO_GRID_LINK");
         c->no_grid_link = gl && gl[0] == '1';
+        const char *cl = std::getenv("RC_NO_CLUSTER");
+        c->no_cluster = cl && cl[0] == '1';
         const char *x = std::getenv("RC_SPLIT");
         c->use_split = x && x[0] == '1';
         const char *y = std::getenv("RC_OWNED");

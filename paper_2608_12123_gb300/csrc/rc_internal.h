@@ -104,6 +104,12 @@ bool chain_grid_tma_plan(int state_bytes, int payload_bytes, uint32_t K, uint32_
 cudaError_t launch_chain_grid_tma(const StepArgs &a, int state_bytes, int payload_bytes, int grid, uint32_t threads,
                                   size_t smem, const void *shape, cudaStream_t s);
 
+// Cluster chain for 512 < K <= 8,192: one cluster of ceil(K / 512) CTAs with
+// the hardware cluster barrier per step.
+bool chain_cluster_plan(int state_bytes, int payload_bytes, uint32_t K, uint32_t *cluster, uint32_t *threads);
+cudaError_t launch_chain_cluster(const StepArgs &a, int state_bytes, int payload_bytes, uint32_t cluster,
+                                 uint32_t threads, cudaStream_t s);
+
 // Grid chain split by links (explicit indices, K a multiple of 8): plan
 // fills 48 bytes of opaque shape and the scratch size (cohort bitmaps and
 // link words); launch clears the bitmaps, marks them, derives the links and

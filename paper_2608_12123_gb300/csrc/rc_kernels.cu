@@ -1743,6 +1743,79 @@ __global__ void __launch_bounds__(544, 1)
 }
 
 // ---------------------------------------------------------------------------
+// Persistent chain, one thread-block cluster (512 < K <= 8,192): C <= 16 CTAs
+// of up to 512 threads, member m = rank * blockDim.x + threadIdx.x.  The step
+// barrier is the cluster's hardware barrier (arrive with release, wait with
+// acquire, cluster scope), not a spin on a global word: each CTA leaves its
+// odd count in its own shared memory, and after the barrier every warp sums
+// the C counts through distributed shared memory.  Records are read at L2
+// (another CTA of the cluster may have stored them the step before; the
+// barrier's release / acquire orders those stores before these loads).
+// Events of the next two steps are prefetched into registers, as in
+// k_chain_cta.  The hardware barrier needs no bounded wait: the CTAs of a
+// cluster are co-scheduled and every one reaches every barrier.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ uint32_t cluster_size() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ void cluster_barrier() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// 32-bit load of the same shared variable in CTA `rank` of the cluster
+__device__ __forceinline__ uint32_t ld_cluster_u32(const uint32_t *p, uint32_t rank) {
+    uint32_t remote, v;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_addr(p)), "r"(rank));
+    asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(v) : "r"(remote) : "memory");
+    return v;
+}
+
+template <int SB, int P>
+__global__ void __launch_bounds__(512) k_chain_cluster(StepArgs a) {
+    __shared__ __align__(16) uint8_t tab[2 * 256 * 8];
+    __shared__ uint32_t cnt[2];
+    const uint32_t tid = threadIdx.x;
+    const uint32_t rank = cluster_rank();
+    const uint32_t C = cluster_size();
+    const uint32_t m = rank * blockDim.x + tid;
+    const bool active = m < a.K;
+    const uint32_t lane = tid & 31u;
+    stage_tables(tab, a.tables, a.tab_stride, 2, 0);
+    uint32_t sel = ld_volatile_u32(&a.dev->sel) & 1u;
+    Event<P> ev0, ev1;
+    if (active && a.n_steps > 0) load_event<P>(ev0, a, 0, m);
+    if (active && a.n_steps > 1) load_event<P>(ev1, a, 1 % a.n_sets, m);
+    cluster_barrier();  // every CTA's tables and counters are in place
+    for (uint32_t n = 0; n < a.n_steps; ++n) {
+        uint32_t odd = 0;
+        if (active) {
+            const Event<P> ev = ev0;
+            ev0 = ev1;
+            if (n + 2u < a.n_steps) load_event<P>(ev1, a, (n + 2u) % a.n_sets, m);
+            odd = transition<SB, P, true>(a, ev, tab + sel * a.tab_stride, sel, n, m);
+        }
+        const uint32_t c = static_cast<uint32_t>(__syncthreads_count(odd));
+        if (tid == 0) cnt[n & 1u] = c;
+        cluster_barrier();  // this step's records and counts, cluster-wide
+        const uint32_t v = lane < C ? ld_cluster_u32(&cnt[n & 1u], lane) : 0u;
+        const uint32_t total = __reduce_add_sync(0xffffffffu, v);
+        sel = total > a.K / 2u ? 1u : 0u;
+        if (rank == 0 && tid == 0 && a.decisions) a.decisions[n] = sel;
+    }
+    cluster_barrier();  // no CTA leaves while another may still read its counters
+    if (rank == 0 && tid == 0) {
+        if (a.n_steps > 0) a.dev->sel = sel;
+        a.dev->step = a.n_steps;
+    }
+}
+
+// ---------------------------------------------------------------------------
 // Persistent chain, split-phase (explicit session indices, K a multiple of 8,
 // at most 512 members per CTA; one CTA when K <= 512, else one CTA per SM).
 //
@@ -2881,6 +2954,60 @@ cudaError_t launch_chain_grid_link(const StepArgs &a, int SB, int P, int grid, u
     const uint32_t *l = lnk;
     void *args[] = {&map, &aa, &l, &gs};
     return cudaLaunchCooperativeKernel(grid_link_fn(SB, P), dim3(grid), dim3(threads), args, smem, s);
+}
+
+namespace {
+const void *cluster_fn(int SB, int P) {
+    return dispatch(SB, P, [](auto b, auto q) {
+        return reinterpret_cast<const void *>(&k_chain_cluster<decltype(b)::value, decltype(q)::value>);
+    });
+}
+cudaLaunchConfig_t cluster_cfg(uint32_t cluster, uint32_t threads, cudaStream_t s, cudaLaunchAttribute *attr) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(cluster);
+    cfg.blockDim = dim3(threads);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = s;
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = cluster;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cfg;
+}
+}  // namespace
+
+// One cluster of C = ceil(K / 512) CTAs (at most 16, a non-portable size
+// above 8); false when the device cannot place such a cluster.
+bool chain_cluster_plan(int SB, int P, uint32_t K, uint32_t *cluster, uint32_t *threads) {
+    if (K <= 512u || K > 8192u) return false;
+    const uint32_t C = (K + 511u) / 512u;
+    const uint32_t T = ((K + C - 1u) / C + 31u) / 32u * 32u;
+    const void *fn = cluster_fn(SB, P);
+    if (C > 8u && cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    cudaLaunchAttribute attr[1];
+    cudaLaunchConfig_t cfg = cluster_cfg(C, T, nullptr, attr);
+    int n_clusters = 0;
+    if (cudaOccupancyMaxActiveClusters(&n_clusters, fn, &cfg) != cudaSuccess || n_clusters < 1) {
+        cudaGetLastError();
+        return false;
+    }
+    *cluster = C;
+    *threads = T;
+    return true;
+}
+
+cudaError_t launch_chain_cluster(const StepArgs &a, int SB, int P, uint32_t cluster, uint32_t threads,
+                                 cudaStream_t s) {
+    cudaLaunchAttribute attr[1];
+    cudaLaunchConfig_t cfg = cluster_cfg(cluster, threads, s, attr);
+    StepArgs aa = a;
+    void *args[] = {&aa};
+    return cudaLaunchKernelExC(&cfg, cluster_fn(SB, P), args);
 }
 
 static const void *split_fn(int SB, int P) {

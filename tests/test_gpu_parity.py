@@ -286,3 +286,21 @@ def test_linked_single_cta_ring_wraps(g, rc, SB, P, K, extra, want_launches, n_s
         assert launches == want_launches
     finally:
         rc.rc_free(ctx)
+
+
+@pytest.mark.parametrize("cluster", [True, False])
+@pytest.mark.parametrize("SB,P", [(16, 64), (64, 128), (16, 32)])
+@pytest.mark.parametrize("K,extra,identity", [(513, 7, False), (1024, 0, False), (4100, 31, False), (8192, 5, False),
+                                              (2048, 0, True)])
+def test_cluster_chain(g, rc, monkeypatch, cluster, SB, P, K, extra, identity):
+    """512 < K <= 8,192: one thread-block cluster (up to 16 CTAs) with the
+    hardware cluster barrier, against the oracle; sessions drawn from K + extra
+    so that most recur in the next step in another CTA of the cluster.  The
+    grid kernels (cluster off) on the same inputs as a control."""
+    monkeypatch.setenv("RC_NO_CLUSTER", "0" if cluster else "1")
+    S = 256 if SB == 64 else 64
+    tables, state0, outc, pay, idx = _inputs(110 + K % 13, K, S, SB, P, 5, N=None if identity else K + extra)
+    n = 11
+    want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=1)
+    got = g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K, sel0=1)
+    g.assert_same(got, want, f"cluster={cluster} K={K} SB={SB} P={P}")
