@@ -592,8 +592,62 @@ def sweep(args):
         if all(per_k[str(k2)]["gpu_resident_us"] < per_k[str(k2)]["cpu_oracle_us"] for k2 in ks[i:]):
             k_r = k
             break
+    # per-route compaction: R routes of K = 256 members each per step, one
+    # segmented launch (rc_seg_step) against one rc_cohort_step per route
+    seg = {}
+    K = 256
+    for R in (1, 4, 16, 64):
+        N = 4 * R * K
+        steps = 16
+        tabs = np.stack([wl.make_tables(S, wl.stream_seed(21, wl.Purpose.TABLE, r)) for r in range(R)])
+        outc, pay, _ = wl.make_cohort_events(21, steps, R * K, P)
+        idx = np.stack([wl.sample_without_replacement(N, R * K, wl.stream_seed(21, wl.Purpose.INDEX, j))
+                        for j in range(steps)]).astype(np.uint32)
+        state = torch.from_numpy(wl.make_state(N, S, SB, wl.stream_seed(21, wl.Purpose.STATE))).cuda()
+        o_d = torch.from_numpy(outc.view(np.int32)).cuda()
+        p_d = torch.from_numpy(pay).cuda()
+        i_d = torch.from_numpy(idx.view(np.int32)).cuda()
+        eff = torch.empty(R * K * 16, dtype=torch.uint8, device="cuda")
+        routes = np.arange(R, dtype=np.uint32)
+        off = (np.arange(R + 1) * K).astype(np.uint32)
+        sctx = rc.rc_seg_init(R, S, tabs, SB, P, R * K, R, N, stream)
+        evs = [rc.make_events(o_d[j], p_d[j], i_d[j], payload_bytes=P, n_sets=1) for j in range(steps)]
+        ctxs = [rc.rc_init(S, tabs[r], SB, P, K, N, stream) for r in range(R)]
+        evr = [[rc.make_events(o_d[j, r * K:(r + 1) * K], p_d[j, r * K:(r + 1) * K], i_d[j, r * K:(r + 1) * K],
+                               payload_bytes=P, n_sets=1) for r in range(R)] for j in range(steps)]
+
+        def timed(fn, n=200):
+            for j in range(10):
+                fn(j)
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for j in range(n):
+                fn(j)
+            e1.record(stream)
+            e1.synchronize()
+            return e0.elapsed_time(e1) * 1000.0 / n
+
+        def one_launch(j):
+            rc.rc_seg_step(sctx, state, evs[j % steps], routes, off, None, eff)
+
+        def per_route(j):
+            for r in range(R):
+                rc.rc_cohort_step(ctxs[r], state, evr[j % steps][r], K, 0, eff[r * K * 16:(r + 1) * K * 16])
+
+        a = timed(one_launch)
+        rc.rc_seg_sync(sctx)
+        b = timed(per_route)
+        for cx in ctxs:
+            rc.rc_sync(cx)
+            rc.rc_free(cx)
+        rc.rc_seg_free(sctx)
+        seg[str(R)] = {"one_segmented_launch_us_per_step": round(a, 3), "one_launch_per_route_us_per_step": round(b, 3),
+                       "ratio": round(b / a, 3)}
+
     return {"sweep": {"workload": "cohorts of N distinct sessions out of 4N, 16-byte state, 64-byte payload, "
                                   "S=64, ring of 64 cohorts; medians of repeated calls",
+                      "segmented_routes_K256": seg,
                       "horizon_us_per_call": horizon, "ratio_host_rt_over_resident": ratio,
                       "safe_suffix": {"per_K_us_per_invocation": per_k, "K_r": k_r,
                                       "cpu": "oracle chain, one thread, 16 steps per K"}}}

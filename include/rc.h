@@ -255,6 +255,41 @@ int64_t rc_former_pop_many(rc_former *f, uint64_t max_cohorts, int64_t *members_
 int rc_former_counts(rc_former *f, int64_t *pushed, int64_t *launched, int64_t *fallback);
 int rc_former_free(rc_former *f);
 
+/* Segmented step: one launch over several route-keyed cohorts (per-route
+ * compaction with variable route bodies; Section 9.1 describes the route
+ * service, and the scope paragraph of Section 10 lists what a single global
+ * decision leaves out).  A context holds n_routes routes, each with its own
+ * pair of bodies (tables: host [n_routes][2][S][8], entries < S; body A then
+ * B) and its own decision flag (0 after rc_seg_init), resident in device
+ * memory.  rc_seg_step transitions, in one launch, n_segments cohorts given
+ * back to back in one event set: segment g holds members [seg_off[g],
+ * seg_off[g+1]) of route seg_route[g].  Each member transitions as in
+ * rc_cohort_step with its route's body T_r selected by flag[r]; then for
+ * every segment d_g = (odd route keys in g) > floor(size_g / 2) (0 for an
+ * empty segment) becomes flag[seg_route[g]] and decisions_out[g].
+ * Contract: seg_route and seg_off are host arrays (n_segments and
+ * n_segments + 1 words; seg_off[0] = 0, non-decreasing, total <=
+ * max_members); a route appears at most once per step; sessions are distinct
+ * across the whole step, so the segments commute.  state, events,
+ * decisions_out (device, [n_segments] u32 or NULL) and effects_out (device,
+ * [total][16] or NULL) as in rc_cohort_step.  Asynchronous on the context
+ * stream; rc_seg_sync waits and returns a latched error (state >= S or
+ * outcome >= 8: RC_E_STATE; index >= n_sessions: RC_E_INDEX; the text names
+ * the segment and member).  RC_E_INVAL for a layout that breaks the
+ * contract (nothing launched).                                              */
+typedef struct rc_seg rc_seg;
+int rc_seg_init(rc_seg **out, uint32_t n_routes, uint32_t S, const uint8_t *tables, uint32_t state_bytes,
+                uint32_t payload_bytes, uint32_t max_members, uint32_t max_segments, uint64_t n_sessions,
+                void *cuda_stream);
+int rc_seg_step(rc_seg *ctx, void *state, const rc_events *events, uint32_t n_segments, const uint32_t *seg_route,
+                const uint32_t *seg_off, uint32_t *decisions_out, void *effects_out);
+int rc_seg_sync(rc_seg *ctx);
+/* Flags of all routes (host [n_routes]); both synchronise. */
+int rc_seg_get_flags(rc_seg *ctx, uint32_t *flags_out);
+int rc_seg_set_flags(rc_seg *ctx, const uint32_t *flags);
+const char *rc_seg_last_error(rc_seg *ctx);
+int rc_seg_free(rc_seg *ctx);
+
 /* Opportunity counts of an event set (host, Section 4), at threshold K and
  * deadline delta_ns for every route:
  *   fixed  events in (route, window) buckets holding >= K events, windows

@@ -44,7 +44,9 @@ MECHANISMS = {"host_rt": RC_MECH_HOST_RT, "resident_cond": RC_MECH_RESIDENT_COND
 EXPORTS = ("rc_init", "rc_cohort_step", "rc_chain", "rc_free", "rc_last_error", "rc_sync",
            "rc_get_decision", "rc_set_decision", "rc_set_wait_limits", "rc_launch_floor",
            "rc_debug_skip_arrival", "rc_last_chain_stats", "rc_set_trace", "rc_cohort_step_noalloc", "rc_former_create", "rc_former_push", "rc_former_pop",
-           "rc_former_push_many", "rc_former_pop_many", "rc_former_counts", "rc_former_free", "rc_opportunity")
+           "rc_former_push_many", "rc_former_pop_many", "rc_former_counts", "rc_former_free", "rc_opportunity",
+           "rc_seg_init", "rc_seg_step", "rc_seg_sync", "rc_seg_get_flags", "rc_seg_set_flags", "rc_seg_last_error",
+           "rc_seg_free")
 
 
 class rc_opportunity_counts(C.Structure):
@@ -86,6 +88,13 @@ def _load():
         "rc_former_counts": (i, [vp, P(i64), P(i64), P(i64)]),
         "rc_former_free": (i, [vp]),
         "rc_opportunity": (i, [vp, vp, u64, u32, u32, i64, i64, P(rc_opportunity_counts)]),
+        "rc_seg_init": (i, [P(vp), u32, u32, vp, u32, u32, u32, u32, u64, vp]),
+        "rc_seg_step": (i, [vp, vp, P(rc_events), u32, vp, vp, vp, vp]),
+        "rc_seg_sync": (i, [vp]),
+        "rc_seg_get_flags": (i, [vp, vp]),
+        "rc_seg_set_flags": (i, [vp, vp]),
+        "rc_seg_last_error": (C.c_char_p, [vp]),
+        "rc_seg_free": (i, [vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -344,3 +353,67 @@ def opportunity_shares(t_ns, route, n_routes, K, delta_ns, launched, origin_ns=0
     out["G"] = (p - f) / (u - f) if u > f else None
     out["R_A"] = (launched - f) / (p - f) if p > f else None
     return out
+
+
+class SegCtx:
+    """A segmented-step context (rc_seg_*): n_routes routes, each with its own
+    pair of bodies and its own device-resident flag."""
+
+    def __init__(self, handle, n_routes):
+        self.handle = handle
+        self.n_routes = n_routes
+
+
+def _seg_check(ctx, rc):
+    if rc != RC_OK:
+        msg = _lib.rc_seg_last_error(ctx.handle) if ctx and ctx.handle else b""
+        raise RcError(rc, msg.decode() if msg else "")
+
+
+def rc_seg_init(n_routes, S, tables, state_bytes, payload_bytes, max_members, max_segments, n_sessions, stream=None):
+    """tables: uint8 [n_routes][2][S][8] (body A then B per route)."""
+    import numpy as np
+    tables = np.ascontiguousarray(tables, dtype=np.uint8)
+    if tables.size != n_routes * 2 * S * 8:
+        raise ValueError("tables must hold n_routes x 2 x S x 8 entries")
+    h = C.c_void_p()
+    st = None if stream is None else (stream if isinstance(stream, int) else int(stream.cuda_stream))
+    rc = _lib.rc_seg_init(C.byref(h), n_routes, S, tables.ctypes.data, state_bytes, payload_bytes, max_members,
+                          max_segments, n_sessions, st)
+    if rc != RC_OK:
+        raise RcError(rc, "rc_seg_init failed")
+    return SegCtx(h.value, n_routes)
+
+
+def rc_seg_step(ctx, state, events, seg_route, seg_off, decisions=None, effects=None):
+    """seg_route, seg_off: host integer arrays (n and n + 1 entries)."""
+    import numpy as np
+    seg_route = np.ascontiguousarray(seg_route, dtype=np.uint32)
+    seg_off = np.ascontiguousarray(seg_off, dtype=np.uint32)
+    if len(seg_off) != len(seg_route) + 1:
+        raise ValueError("seg_off needs one entry more than seg_route")
+    _seg_check(ctx, _lib.rc_seg_step(ctx.handle, _ptr(state), C.byref(events), len(seg_route), seg_route.ctypes.data,
+                                     seg_off.ctypes.data, _ptr(decisions), _ptr(effects)))
+
+
+def rc_seg_sync(ctx):
+    _seg_check(ctx, _lib.rc_seg_sync(ctx.handle))
+
+
+def rc_seg_get_flags(ctx):
+    import numpy as np
+    out = np.zeros(ctx.n_routes, dtype=np.uint32)
+    _seg_check(ctx, _lib.rc_seg_get_flags(ctx.handle, out.ctypes.data))
+    return out
+
+
+def rc_seg_set_flags(ctx, flags):
+    import numpy as np
+    flags = np.ascontiguousarray(flags, dtype=np.uint32)
+    _seg_check(ctx, _lib.rc_seg_set_flags(ctx.handle, flags.ctypes.data))
+
+
+def rc_seg_free(ctx):
+    if ctx and ctx.handle:
+        _lib.rc_seg_free(ctx.handle)
+        ctx.handle = None

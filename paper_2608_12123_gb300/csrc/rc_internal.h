@@ -50,6 +50,32 @@ struct StepArgs {
     long long *trace;        // optional per-step phase clocks of two CTAs (profiling), or null
 };
 
+// A segmented step (rc_seg_step): n_seg route-keyed cohorts concatenated;
+// segment g holds members [seg_off[g], seg_off[g+1]) and uses route
+// seg_route[g], whose bodies are tables + (2 route + sel) * tab_stride and
+// whose flag is flags[route].  count (n_seg words) and ticket start at zero
+// and are left at zero.
+struct SegArgs {
+    uint8_t *state;
+    uint64_t n_sessions;
+    const uint32_t *outcome;
+    const uint8_t *payload;
+    const uint32_t *idx;  // null: member m is session m
+    uint32_t total;
+    uint32_t n_seg;
+    const uint32_t *seg_route;
+    const uint32_t *seg_off;
+    const uint8_t *tables;
+    uint32_t S;
+    uint32_t tab_stride;
+    uint32_t *flags;
+    uint32_t *count;
+    uint32_t *ticket;
+    uint32_t *decisions;  // [n_seg] or null
+    uint8_t *effects;     // [total][16] or null
+    DevBlock *dev;
+};
+
 // Epilogue flags of the per-step kernel.
 enum : uint32_t {
     EPI_NONE = 0u,
@@ -144,6 +170,9 @@ cudaError_t launch_chain_owned(const StepArgs &a, int state_bytes, int payload_b
                                size_t smem, const void *shape, const uint32_t *perm_m, const uint32_t *perm_s,
                                const uint32_t *perm_o, const uint32_t *off, const uint8_t *pay_routed,
                                cudaStream_t s);
+
+// One segmented step (at least one CTA, so that empty segments decide 0).
+cudaError_t launch_seg_step(const SegArgs &a, int state_bytes, int payload_bytes, cudaStream_t s);
 
 // Writes decisions[0..n) = 0 and sel = 0 (an empty cohort decides 0).
 cudaError_t launch_empty_cohorts(const StepArgs &a, cudaStream_t s);

@@ -2526,6 +2526,99 @@ __global__ void __launch_bounds__(512, 1)
     }
 }
 
+// ---------------------------------------------------------------------------
+// Segmented step: one launch over several route-keyed cohorts (segments),
+// each with its own pair of route bodies and its own decision chain (the
+// per-route compaction with variable route bodies that Section 9.1 and the
+// scope paragraph of Section 10 leave to a route service).  Member m finds
+// its segment by binary search over seg_off, transitions with the body its
+// route's flag selects, and adds its odd key to its segment's count (warp
+// lanes of one segment aggregate first); the last CTA (ticket) turns every
+// count into that segment's decision, the route's next flag.  Sessions are
+// distinct across the whole step (checked by the caller's contract), so the
+// segments commute and the step equals their cohort steps in any order.
+// ---------------------------------------------------------------------------
+template <int SB, int P>
+__global__ void __launch_bounds__(kStepThreads) k_seg_step(SegArgs a) {
+    constexpr int NV = SB / 16;
+    __shared__ uint32_t s_last;
+    const uint32_t tid = threadIdx.x;
+    const uint32_t lane = tid & 31u;
+    const uint32_t m = blockIdx.x * blockDim.x + tid;
+    const bool act = m < a.total;
+    uint32_t g = 0, odd = 0;
+    if (act) {
+        uint32_t lo = 0, hi = a.n_seg;  // seg_off[lo] <= m < seg_off[hi]
+        while (hi - lo > 1u) {
+            const uint32_t mid = (lo + hi) >> 1;
+            if (__ldg(a.seg_off + mid) <= m) lo = mid;
+            else hi = mid;
+        }
+        g = lo;
+        const uint32_t r = __ldg(a.seg_route + g);
+        const uint32_t sel = a.flags[r] & 1u;
+        const uint8_t *tab = a.tables + static_cast<size_t>(2u * r + sel) * a.tab_stride;
+        const uint32_t s = a.idx ? __ldg(a.idx + m) : m;
+        const uint32_t o = __ldg(a.outcome + m);
+        if (s >= a.n_sessions) {
+            latch_error(a.dev, DEV_E_INDEX, g, m);
+        } else {
+            uint4 *rp = reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(s) * SB);
+            uint4 rr[NV];
+#pragma unroll
+            for (int k = 0; k < NV; ++k) rr[k] = rp[k];
+            const uint32_t x = rr[0].x;
+            if (x >= a.S || o >= 8u) {
+                latch_error(a.dev, DEV_E_STATE, g, m);
+            } else {
+                uint4 pw[P / 16];
+                const uint4 *src = reinterpret_cast<const uint4 *>(a.payload + static_cast<size_t>(m) * P);
+#pragma unroll
+                for (int k = 0; k < P / 16; ++k) pw[k] = __ldg(src + k);
+                const uint64_t rk = route_key<P>(x, o, pw);
+                const uint32_t y = __ldg(tab + x * 8u + o);
+                rr[0].x = y;
+                rr[0].y = rr[0].y + 1u;
+                mix_acc<SB>(rr, rk);
+#pragma unroll
+                for (int k = 0; k < NV; ++k) rp[k] = rr[k];
+                if (a.effects) {
+                    uint4 e;
+                    e.x = static_cast<uint32_t>(rk);
+                    e.y = static_cast<uint32_t>(rk >> 32);
+                    e.z = s;
+                    e.w = y | (o << 16) | (sel << 24);
+                    __stcs(reinterpret_cast<uint4 *>(a.effects) + m, e);
+                }
+                odd = static_cast<uint32_t>(rk & 1u);
+            }
+        }
+    }
+    // per-segment odd counts: lanes of one segment aggregate, their first lane adds
+    const uint32_t amask = __ballot_sync(0xffffffffu, act);
+    if (act) {
+        const uint32_t same = __match_any_sync(amask, g);
+        const uint32_t c = __popc(__ballot_sync(amask, odd != 0u) & same);
+        if (lane == static_cast<uint32_t>(__ffs(same) - 1) && c != 0u) atomicAdd(a.count + g, c);
+    }
+    __syncthreads();
+    if (tid == 0) {
+        __threadfence();
+        s_last = atomicAdd(a.ticket, 1u) == gridDim.x - 1u ? 1u : 0u;
+    }
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    for (uint32_t q = tid; q < a.n_seg; q += blockDim.x) {
+        const uint32_t c = atomicExch(a.count + q, 0u);
+        const uint32_t size = __ldg(a.seg_off + q + 1u) - __ldg(a.seg_off + q);
+        const uint32_t d = c > size / 2u ? 1u : 0u;
+        a.flags[__ldg(a.seg_route + q)] = d;
+        if (a.decisions) a.decisions[q] = d;
+    }
+    if (tid == 0) *a.ticket = 0u;
+}
+
 __global__ void k_empty_cohorts(StepArgs a) {
     for (uint32_t n = blockIdx.x * blockDim.x + threadIdx.x; n < a.n_steps; n += gridDim.x * blockDim.x)
         if (a.decisions) a.decisions[n] = 0u;
@@ -3175,6 +3268,16 @@ cudaError_t launch_chain_owned(const StepArgs &a, int SB, int P, int grid, uint3
     OwnedShape shc = sh;
     void *args[] = {&map, &aa, &shc, &perm_m, &perm_s, &perm_o, &off};
     return cudaLaunchCooperativeKernel(owned_fn(SB, P, sh.res != 0), dim3(grid), dim3(threads), args, smem, s);
+}
+
+cudaError_t launch_seg_step(const SegArgs &a, int SB, int P, cudaStream_t s) {
+    const void *fn = dispatch(SB, P, [](auto b, auto q) {
+        return reinterpret_cast<const void *>(&k_seg_step<decltype(b)::value, decltype(q)::value>);
+    });
+    SegArgs aa = a;
+    void *args[] = {&aa};
+    const uint32_t grid = a.total == 0u ? 1u : (a.total + kStepThreads - 1u) / kStepThreads;
+    return cudaLaunchKernel(fn, dim3(grid), dim3(kStepThreads), args, 0, s);
 }
 
 cudaError_t launch_empty_cohorts(const StepArgs &a, cudaStream_t s) {
