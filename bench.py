@@ -645,8 +645,51 @@ def sweep(args):
         seg[str(R)] = {"one_segmented_launch_us_per_step": round(a, 3), "one_launch_per_route_us_per_step": round(b, 3),
                        "ratio": round(b / a, 3)}
 
+    # the exact-packing grid of Section 5.2 on the GPU: C x seed swarms, three
+    # groupings, deadlines x thresholds per swarm and grouping (540 rows)
+    panel = wl.make_panel()
+    ks = [32, 64, 128, 256]
+    ds = [10_000_000, 25_000_000, 50_000_000, 100_000_000, 250_000_000]
+    grid_rows, gpu_s, gen_s, prop1 = 0, 0.0, 0.0, True
+    at = {}
+    host_row_s = None
+    for C in (1_000, 10_000, 100_000):
+        acc = {}
+        for seed in range(3):
+            t0 = time.perf_counter()
+            arr = wl.make_arrivals(C, panel, seed_index=seed)
+            gen_s += time.perf_counter() - t0
+            for grouping, route, R in (("route_key", arr.route, panel.n_labels),
+                                       ("event_class", (arr.route % 8).astype(np.uint32), 8),
+                                       ("pooled", np.zeros(arr.n, np.uint32), 1)):
+                t0 = time.perf_counter()
+                cnt = rc.rc_opportunity_grid(arr.t_ns, route, R, ks, ds, 0, stream)
+                gpu_s += time.perf_counter() - t0
+                grid_rows += len(ks) * len(ds)
+                f, pst, u = cnt[..., 0].astype(np.int64), cnt[..., 1].astype(np.int64), cnt[..., 2].astype(np.int64)
+                prop1 = prop1 and bool(np.all(f <= pst) and np.all(pst <= u))
+                fx, px, ux = (int(v) for v in cnt[2, 3])  # delta 50 ms, K 256
+                g_ = (px - fx) / (ux - fx) if ux > fx else None
+                a_ = acc.setdefault(grouping, {"F": [], "P_star": [], "U": [], "G": []})
+                for key, v in (("F", fx / arr.n), ("P_star", px / arr.n), ("U", ux / arr.n), ("G", g_)):
+                    if v is not None:
+                        a_[key].append(v)
+                if C == 100_000 and seed == 0 and grouping == "route_key":
+                    t0 = time.perf_counter()
+                    rc.rc_opportunity(arr.t_ns, route, R, 256, 50_000_000, 0)
+                    host_row_s = time.perf_counter() - t0
+        at[str(C)] = {gk: {k: (round(float(np.mean(v)), 5) if v else None) for k, v in gv.items()}
+                      for gk, gv in acc.items()}
+    opp_grid = {"rows": grid_rows, "gpu_call_seconds": round(gpu_s, 3), "arrival_generation_seconds": round(gen_s, 3),
+                "F_le_Pstar_le_U_every_row": prop1,
+                "host_rc_opportunity_seconds_one_row_C100k": None if host_row_s is None else round(host_row_s, 3),
+                "mean_over_seeds_delta50ms_K256": at,
+                "grid": "C in {1k, 10k, 100k} x 3 seeds x {route key, event class, pooled} x delta in {10, 25, 50, "
+                        "100, 250} ms x K in {32, 64, 128, 256}"}
+
     return {"sweep": {"workload": "cohorts of N distinct sessions out of 4N, 16-byte state, 64-byte payload, "
                                   "S=64, ring of 64 cohorts; medians of repeated calls",
+                      "opportunity_grid": opp_grid,
                       "segmented_routes_K256": seg,
                       "horizon_us_per_call": horizon, "ratio_host_rt_over_resident": ratio,
                       "safe_suffix": {"per_K_us_per_invocation": per_k, "K_r": k_r,

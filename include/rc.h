@@ -309,6 +309,20 @@ typedef struct {
 int rc_opportunity(const int64_t *t_ns, const uint32_t *route, uint64_t n, uint32_t n_routes, uint32_t K,
                    int64_t delta_ns, int64_t origin_ns, rc_opportunity_counts *out);
 
+/* The same three counts for every (delta, K) pair of a grid, on the GPU (the
+ * exact-packing grid of Section 5.2: deadlines x thresholds per event set and
+ * grouping).  One GPU thread per (route, delta) runs the fixed-window runs
+ * and the U scan for every K, one per (route, delta, K) the P* recurrence,
+ * over that route's times; the host groups the events by route (a counting
+ * pass when they come in time order).  counts_out (host, u64
+ * [n_delta][n_K][3]) receives {fixed, exact, upper} per pair.  Scratch of
+ * 8 n n_delta n_K bytes is allocated and freed inside the call, which
+ * synchronises cuda_stream.  RC_E_INVAL as for rc_opportunity, for n >= 2^31
+ * or n_K > 32; RC_E_NOMEM when the scratch does not fit.                   */
+int rc_opportunity_grid(const int64_t *t_ns, const uint32_t *route, uint64_t n, uint32_t n_routes,
+                        const uint32_t *K_list, uint32_t n_K, const int64_t *delta_list, uint32_t n_delta,
+                        int64_t origin_ns, uint64_t *counts_out, void *cuda_stream);
+
 #ifdef __cplusplus
 }
 #endif

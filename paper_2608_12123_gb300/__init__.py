@@ -46,7 +46,7 @@ EXPORTS = ("rc_init", "rc_cohort_step", "rc_chain", "rc_free", "rc_last_error", 
            "rc_debug_skip_arrival", "rc_last_chain_stats", "rc_set_trace", "rc_cohort_step_noalloc", "rc_former_create", "rc_former_push", "rc_former_pop",
            "rc_former_push_many", "rc_former_pop_many", "rc_former_counts", "rc_former_free", "rc_opportunity",
            "rc_seg_init", "rc_seg_step", "rc_seg_sync", "rc_seg_get_flags", "rc_seg_set_flags", "rc_seg_last_error",
-           "rc_seg_free")
+           "rc_seg_free", "rc_opportunity_grid")
 
 
 class rc_opportunity_counts(C.Structure):
@@ -95,6 +95,7 @@ def _load():
         "rc_seg_set_flags": (i, [vp, vp]),
         "rc_seg_last_error": (C.c_char_p, [vp]),
         "rc_seg_free": (i, [vp]),
+        "rc_opportunity_grid": (i, [vp, vp, u64, u32, vp, u32, vp, u32, i64, vp, vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -417,3 +418,20 @@ def rc_seg_free(ctx):
     if ctx and ctx.handle:
         _lib.rc_seg_free(ctx.handle)
         ctx.handle = None
+
+
+def rc_opportunity_grid(t_ns, route, n_routes, K_list, delta_list, origin_ns=0, stream=None):
+    """{fixed, exact, upper} for every (delta, K) pair, on the GPU: returns a
+    uint64 array [len(delta_list)][len(K_list)][3]."""
+    import numpy as np
+    t_ns = np.ascontiguousarray(t_ns, dtype=np.int64)
+    route = np.ascontiguousarray(route, dtype=np.uint32)
+    ks = np.ascontiguousarray(K_list, dtype=np.uint32)
+    ds = np.ascontiguousarray(delta_list, dtype=np.int64)
+    out = np.zeros((len(ds), len(ks), 3), dtype=np.uint64)
+    st = None if stream is None else (stream if isinstance(stream, int) else int(stream.cuda_stream))
+    rc = _lib.rc_opportunity_grid(t_ns.ctypes.data, route.ctypes.data, len(t_ns), n_routes, ks.ctypes.data, len(ks),
+                                  ds.ctypes.data, len(ds), origin_ns, out.ctypes.data, st)
+    if rc != RC_OK:
+        raise RcError(rc, "rc_opportunity_grid failed")
+    return out

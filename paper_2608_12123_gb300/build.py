@@ -21,7 +21,7 @@ LIB = os.path.join(OUT_DIR, "librc.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++20", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC,
               "--expt-relaxed-constexpr"]
-CU_SOURCES = ["rc_kernels.cu", "rc_api.cu", "rc_seg.cu"]
+CU_SOURCES = ["rc_kernels.cu", "rc_api.cu", "rc_seg.cu", "rc_grid.cu"]
 CXX_SOURCES = ["rc_former.cpp", "rc_opportunity.cpp"]
 
 
