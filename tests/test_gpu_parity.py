@@ -134,10 +134,11 @@ def test_bad_inputs_are_latched_and_the_context_survives(g, rc):
     g.assert_same(g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K), want, "after errors")
 
 
-def test_grid_barrier_wait_is_bounded(g, rc):
+def test_grid_barrier_wait_is_bounded(g, rc, monkeypatch):
     """A CTA that never arrives (test hook) makes the others' bounded waits run
     out: RC_E_TIMEOUT comes back and the context keeps working."""
     import torch
+    monkeypatch.setenv("RC_NO_CLUSTER", "1")  # the grid kernel, not the cluster one
     K, S, SB, P, n = 4096, 16, 16, 32, 4
     tables, state0, outc, pay, idx = _inputs(17, K, S, SB, P, 2, N=5000)
     ctx = rc.rc_init(S, tables, SB, P, K, 5000, torch.cuda.current_stream())
@@ -187,6 +188,7 @@ def test_persistent_grid_kernels(g, rc, monkeypatch, kernel, SB, P, K, N, identi
     monkeypatch.setenv("RC_SPLIT", "1" if kernel == "split" else "0")
     monkeypatch.setenv("RC_NO_TMA", "1" if kernel == "plain" else "0")
     monkeypatch.setenv("RC_NO_GRID_LINK", "0" if kernel == "link" else "1")
+    monkeypatch.setenv("RC_NO_CLUSTER", "1")  # K <= 8192 would otherwise take the cluster kernel
     S = 256 if SB == 64 else 64
     tables, state0, outc, pay, idx = _inputs(50 + K % 11, K, S, SB, P, 3, N=None if identity else N)
     n = 5
@@ -202,6 +204,7 @@ def test_grid_barrier_wait_is_bounded_every_grid_kernel(g, rc, monkeypatch, kern
     monkeypatch.setenv("RC_SPLIT", "1" if kernel == "split" else "0")
     monkeypatch.setenv("RC_NO_TMA", "1" if kernel == "plain" else "0")
     monkeypatch.setenv("RC_NO_GRID_LINK", "0" if kernel == "link" else "1")
+    monkeypatch.setenv("RC_NO_CLUSTER", "1")  # K <= 8192 would otherwise take the cluster kernel
     K, S, SB, P, n = 8192, 16, 16, 64, 4
     tables, state0, outc, pay, idx = _inputs(19, K, S, SB, P, 2, N=9000)
     ctx = rc.rc_init(S, tables, SB, P, K, 9000, torch.cuda.current_stream())
