@@ -1191,7 +1191,9 @@ __global__ void __launch_bounds__(512, 1) k_chain_cta_link(StepArgs a, const uin
 // k_link), as in k_chain_cta_link.  The decision is the barrier's own count.
 // A producer wait that runs out latches RC_E_TIMEOUT; the CTA stops after
 // that step, the producer first waiting (bounded) for the copies it still
-// has in flight.
+// has in flight.  Trace points (thread 0): 0 region start, 1 record landed,
+// 4 input state read, 5 payload read, 6 key done, 2 transition done, 3 after
+// the barrier.
 // ---------------------------------------------------------------------------
 constexpr uint32_t kProdRW = 6;  // word slots (issued five steps ahead)
 constexpr uint32_t kProdRP = 4;  // payload slots (issued three steps ahead)
@@ -1332,6 +1334,10 @@ __global__ void __launch_bounds__(544, 1)
 #pragma unroll
                     for (int k = 0; k < NV; ++k) r[k] = src[k];
                     const uint32_t x = r[0].x;
+                    if (trace) {
+                        asm volatile("" ::"r"(x));
+                        trace[n * 8 + 4] = clock64();
+                    }
                     if (x >= a.S || o >= 8u) {
                         latch_error(a.dev, DEV_E_STATE, n, m);
                         if (src != mine) {
@@ -1341,7 +1347,15 @@ __global__ void __launch_bounds__(544, 1)
                     } else {
                         uint4 pw[P / 16];
                         read_payload_swizzled<P>(pw, pay + static_cast<size_t>(n % RP) * sh.stage_pay, m);
+                        if (trace) {
+                            asm volatile("" ::"r"(pw[P / 16 - 1].w));
+                            trace[n * 8 + 5] = clock64();
+                        }
                         const uint64_t rk = route_key<P>(x, o, pw);
+                        if (trace) {
+                            asm volatile("" ::"l"(rk));
+                            trace[n * 8 + 6] = clock64();
+                        }
                         const uint32_t y = tab[sel * a.tab_stride + x * 8u + o];
                         r[0].x = y;
                         r[0].y = r[0].y + 1u;
@@ -1370,7 +1384,10 @@ __global__ void __launch_bounds__(544, 1)
                     }
                 }
             }
-            if (trace) trace[n * 8 + 2] = clock64();
+            if (trace) {
+                asm volatile("" ::"r"(odd));
+                trace[n * 8 + 2] = clock64();
+            }
             if (!early) gather(n + 2u);
         }
         // the count of odd keys; the barrier also publishes this step's record
@@ -1393,6 +1410,379 @@ __global__ void __launch_bounds__(544, 1)
         }
     }
     if (tid == 0 && n == nst) {
+        if (nst > 0) a.dev->sel = sel;
+        a.dev->step = nst;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Links of reach kFarD: for member m of cohort j, the distance t (1..kFarD)
+// to the nearest earlier cohort holding the same session (cohorts taken
+// cyclically, as a chain walks them) and its position q there, packed as
+// t << 16 | q; 0 when none of the kFarD cohorts before holds the session or
+// the index is out of range.  One CTA per cohort, one open-addressing table
+// per earlier cohort (K <= 512 keys in 1,024 slots).
+// ---------------------------------------------------------------------------
+constexpr uint32_t kFarD = 5;
+
+__global__ void __launch_bounds__(512) k_link_far(const uint32_t *idx, uint32_t n_sets, uint32_t K, uint64_t N,
+                                                  uint32_t *lnk) {
+    __shared__ uint32_t key[kFarD][kLinkSlots];
+    __shared__ uint16_t pos[kFarD][kLinkSlots];
+    for (uint32_t j = blockIdx.x; j < n_sets; j += gridDim.x) {
+        for (uint32_t i = threadIdx.x; i < kFarD * kLinkSlots; i += blockDim.x) (&key[0][0])[i] = kLinkEmpty;
+        __syncthreads();
+        for (uint32_t t = 0; t < kFarD; ++t) {
+            const uint32_t src =
+                static_cast<uint32_t>((static_cast<uint64_t>(j) + kFarD * static_cast<uint64_t>(n_sets) - 1u - t) %
+                                      n_sets);
+            for (uint32_t m = threadIdx.x; m < K; m += blockDim.x) {
+                const uint32_t s = __ldg(idx + static_cast<size_t>(src) * K + m);
+                if (s >= N) continue;
+                uint32_t h = link_hash(s);
+                for (uint32_t probe = 0; probe < kLinkSlots; ++probe) {
+                    const uint32_t prev = atomicCAS(&key[t][h], kLinkEmpty, s);
+                    if (prev == kLinkEmpty || prev == s) {
+                        pos[t][h] = static_cast<uint16_t>(m);
+                        break;
+                    }
+                    h = (h + 1u) & (kLinkSlots - 1u);
+                }
+            }
+        }
+        __syncthreads();
+        for (uint32_t m = threadIdx.x; m < K; m += blockDim.x) {
+            const uint32_t s = __ldg(idx + static_cast<size_t>(j) * K + m);
+            uint32_t l = 0;
+            if (s < N) {
+                for (uint32_t t = 0; t < kFarD && l == 0u; ++t) {
+                    uint32_t h = link_hash(s);
+                    for (uint32_t probe = 0; probe < kLinkSlots; ++probe) {
+                        const uint32_t k = key[t][h];
+                        if (k == s) {
+                            l = ((t + 1u) << 16) | pos[t][h];
+                            break;
+                        }
+                        if (k == kLinkEmpty) break;
+                        h = (h + 1u) & (kLinkSlots - 1u);
+                    }
+                }
+            }
+            lnk[static_cast<size_t>(j) * K + m] = l;
+        }
+        __syncthreads();
+    }
+}
+
+// Named barrier `id` over `count` threads (a multiple of 32): arrive without
+// waiting, or arrive and wait.
+__device__ __forceinline__ void named_arrive(uint32_t id, uint32_t count) {
+    asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+__device__ __forceinline__ void named_sync(uint32_t id, uint32_t count) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
+// Route key from its first finaliser round h0 = fin64((x | o << 32) ^ gamma),
+// taken from a table: one more round per 64-bit payload word.
+template <int P>
+__device__ __forceinline__ uint64_t route_key_from(uint64_t h, const uint4 (&pw)[P / 16]) {
+#pragma unroll
+    for (int k = 0; k < P / 16; ++k) {
+        h = fin64(h ^ pack64(pw[k].x, pw[k].y));
+        h = fin64(h ^ pack64(pw[k].z, pw[k].w));
+    }
+    return h;
+}
+
+// ---------------------------------------------------------------------------
+// Persistent chain, one CTA, explicit session indices, K a multiple of 8 up
+// to 256, with the route keys on the decision path and the records off it.
+//
+// A key needs the session's state value x (the first word of its record),
+// not the rest of the record.  So x travels on its own: step n leaves, per
+// member, the session's state after the step in a ring Y[n] (the new state,
+// or the old one for a rejected member), and k_link_far gives each member
+// the step (at most kFarD back) and position of its session's previous
+// appearance.  A member of step n takes x from that Y entry or, when its
+// session is not in the kFarD steps before, from its record gathered from
+// HBM three steps ahead.
+//
+// Warps 0 .. ceil(K/32) - 1 (key warps), region n: x; y = T_sel[x][o] into
+// Y[n]; the key from a table of first rounds H0[x][o] and one finaliser
+// round per payload word.  The block barrier then counts the odd keys.
+//
+// The next ceil(K/32) warps (record warps), region n: complete the records
+// of step n - 1 with the keys, new states and decision the key warps left.
+// The input record is the output of the session's previous appearance
+// (record ring, up to kFarD steps back) or the gathered one; the output goes
+// to HBM and to the ring, with the effect.  They also gather, for step n + 3,
+// the records of the members without a link: such a session was last written
+// in step n - 3 or earlier, by region n - 2, which that region's barrier made
+// visible to the CTA.
+//
+// A producer warp streams outcomes, session indices and links (issued six
+// steps ahead) and payload tiles (three ahead), as in k_chain_cta_prod.  The
+// loop runs one region past the last step, in which only the record warps
+// work.  A producer wait that runs out latches RC_E_TIMEOUT; the CTA stops
+// after that region, its record warps first completing the step the key
+// warps finished.  Trace points (thread 0): 0 region start, 1 x ready,
+// 2 key done, 3 after the barrier.
+// ---------------------------------------------------------------------------
+constexpr uint32_t kFarRW = 8;           // word slots (issued six ahead)
+constexpr uint32_t kFarRP = 4;           // payload slots (issued three ahead)
+constexpr uint32_t kFarRR = 10;          // record slots: gather at n - 3 .. last forward at n + 1 + kFarD
+constexpr uint32_t kFarRY = kFarD + 1;   // state-after-step slots
+constexpr uint32_t kFarSkip = 0, kFarRejected = 1, kFarApplied = 2;
+
+template <int SB, int P>
+__global__ void __launch_bounds__(544, 1)
+    k_chain_cta_far(const __grid_constant__ CUtensorMap tmap, StepArgs a, const uint32_t *lnk, LinkShape sh) {
+    constexpr int NV = SB / 16;
+    constexpr uint32_t RW = kFarRW, RP = kFarRP, RR = kFarRR, RY = kFarRY;
+    extern __shared__ uint8_t dsm_raw[];
+    __shared__ __align__(8) uint64_t wbar[RW];
+    __shared__ __align__(8) uint64_t pbar[RP];
+    __shared__ uint32_t s_ab[2];
+    const uint32_t raw = smem_addr(dsm_raw);
+    uint8_t *const base = dsm_raw + (((raw + 1023u) & ~1023u) - raw);
+    const uint32_t K = a.K;
+    const uint32_t Kw = (K + 31u) & ~31u;  // key threads; record threads next, then the producer warp
+    const uint32_t tid = threadIdx.x;
+    const bool keyw = tid < Kw;
+    const bool prod = tid >= 2u * Kw;
+    const uint32_t rt = tid - Kw;  // record-thread member (valid when !keyw && !prod)
+    const uint32_t nst = a.n_steps;
+    const uint64_t limit = a.dev->wait_ns;
+    // layout: [payload slots][records][H0][rk][words][Y][flags][tables]
+    uint8_t *const pay = base;
+    uint4 *const rec = reinterpret_cast<uint4 *>(base + static_cast<size_t>(RP) * sh.stage_pay);  // [RR][K][NV]
+    uint64_t *const h0 = reinterpret_cast<uint64_t *>(rec + static_cast<size_t>(RR) * K * NV);      // [S][8]
+    uint64_t *const rks = h0 + static_cast<size_t>(a.S) * 8u;                                       // [2][K]
+    uint32_t *const words = reinterpret_cast<uint32_t *>(rks + 2u * K);                           // [RW][3][K]
+    uint32_t *const ys = words + static_cast<size_t>(RW) * 3 * K;                                  // [RY][K]
+    uint32_t *const fls = ys + static_cast<size_t>(RY) * K;                                        // [2][K]
+    uint8_t *const tab = reinterpret_cast<uint8_t *>(fls + 2u * K);
+    auto word_of = [&](uint32_t j, uint32_t which) { return words + (static_cast<size_t>(j % RW) * 3 + which) * K; };
+    auto rec_of = [&](uint32_t j, uint32_t m) { return rec + (static_cast<size_t>(j % RR) * K + m) * NV; };
+    const uint64_t stream_pol = policy_evict_first();
+    long long *trace = (a.trace && tid == 0) ? a.trace : nullptr;
+
+    // producer lane 0 only
+    auto issue_words = [&](uint32_t j) {
+        if (j >= nst) return;
+        const size_t e0 = static_cast<size_t>(j % a.n_sets) * K;
+        uint64_t *b = &wbar[j % RW];
+        mbar_arrive_expect_tx(b, 3u * K * 4u);
+        bulk_load_hint(word_of(j, 0), a.outcome + e0, K * 4u, b, stream_pol);
+        bulk_load_hint(word_of(j, 1), a.idx + e0, K * 4u, b, stream_pol);
+        bulk_load_hint(word_of(j, 2), lnk + e0, K * 4u, b, stream_pol);
+    };
+    auto issue_pay = [&](uint32_t j) {
+        if (j >= nst) return;
+        const uint32_t st = j % RP;
+        const int32_t row0 = static_cast<int32_t>((j % a.n_sets) * K);
+        mbar_arrive_expect_tx(&pbar[st], sh.n_boxes * sh.box_rows * P);
+        for (uint32_t b = 0; b < sh.n_boxes; ++b)
+            tma_load_2d_hint(pay + static_cast<size_t>(st) * sh.stage_pay + b * sh.box_rows * P, &tmap, 0,
+                             row0 + static_cast<int32_t>(b * sh.box_rows), &pbar[st], stream_pol);
+    };
+    auto landed_words = [&](uint32_t j) { return j >= nst || mbar_wait_bounded(&wbar[j % RW], (j / RW) & 1u, limit); };
+    auto landed_pay = [&](uint32_t j) { return j >= nst || mbar_wait_bounded(&pbar[j % RP], (j / RP) & 1u, limit); };
+    // a member of step j without a usable link: its record comes from HBM
+    auto unlinked = [](uint32_t l, uint32_t j) {
+        const uint32_t t = l >> 16;
+        return t == 0u || t > j;
+    };
+    // record thread: gather its member's record of step j when unlinked (one
+    // commit group, empty when there is nothing to copy)
+    auto gather = [&](uint32_t j) {
+        if (j < nst && rt < K) {
+            const uint32_t s = word_of(j, 1)[rt];
+            if (s < a.n_sessions && unlinked(word_of(j, 2)[rt], j)) {
+                const uint4 *rp = reinterpret_cast<const uint4 *>(a.state + static_cast<size_t>(s) * SB);
+                uint4 *dst = rec_of(j, rt);
+#pragma unroll
+                for (int k = 0; k < NV; ++k) cp_async16(dst + k, rp + k);
+            }
+        }
+        cp_async_commit();
+    };
+    // record thread: complete its member's record of step j (decision sel_j)
+    auto record_step = [&](uint32_t j, uint32_t sel_j) {
+        if (rt >= K) return;
+        const uint32_t f = fls[(j & 1u) * K + rt];
+        if (f == kFarSkip) return;
+        const uint32_t l = word_of(j, 2)[rt];
+        uint4 *mine = rec_of(j, rt);
+        const uint4 *src = unlinked(l, j) ? mine : rec_of(j - (l >> 16), l & 0xFFFFu);
+        uint4 r[NV];
+#pragma unroll
+        for (int k = 0; k < NV; ++k) r[k] = src[k];
+        if (f == kFarRejected) {
+            if (src != mine) {
+#pragma unroll
+                for (int k = 0; k < NV; ++k) mine[k] = r[k];
+            }
+            return;
+        }
+        const uint32_t o = word_of(j, 0)[rt];
+        const uint32_t s = word_of(j, 1)[rt];
+        const uint32_t y = ys[(j % RY) * K + rt];
+        const uint64_t rk = rks[(j & 1u) * K + rt];
+        r[0].x = y;
+        r[0].y = r[0].y + 1u;
+        mix_acc<SB>(r, rk);
+        uint4 *rp = reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(s) * SB);
+#pragma unroll
+        for (int k = 0; k < NV; ++k) {
+            mine[k] = r[k];
+            rp[k] = r[k];
+        }
+        const size_t slot = static_cast<size_t>(j) * K + rt;
+        if (a.effects) {
+            uint4 e;
+            e.x = static_cast<uint32_t>(rk);
+            e.y = static_cast<uint32_t>(rk >> 32);
+            e.z = s;
+            e.w = y | (o << 16) | (sel_j << 24);
+            __stcs(reinterpret_cast<uint4 *>(a.effects) + slot, e);
+        }
+        if (a.state_log) {
+            uint4 *lp = reinterpret_cast<uint4 *>(a.state_log + slot * SB);
+#pragma unroll
+            for (int k = 0; k < NV; ++k) __stcs(lp + k, r[k]);
+        }
+    };
+
+    if (tid == 0) {
+        for (uint32_t i = 0; i < RW; ++i) mbar_init(&wbar[i], 1);
+        for (uint32_t i = 0; i < RP; ++i) mbar_init(&pbar[i], 1);
+        fence_mbar_init();
+        s_ab[0] = 0;
+        s_ab[1] = 0;
+    }
+    stage_tables(tab, a.tables, a.tab_stride, 2, 0);
+    for (uint32_t i = tid; i < a.S * 8u; i += blockDim.x) h0[i] = fin64(pack64(i >> 3, i & 7u) ^ kGamma);
+    uint32_t sel = ld_volatile_u32(&a.dev->sel) & 1u;
+    uint32_t sel_prev = sel;
+    __syncthreads();
+    // prologue: runs of steps 0..6 and tiles of steps 0..2 go out; the runs
+    // of steps 0..3 and the tiles of step 0 are waited for; the record warps
+    // then gather steps 0, 1 and 2 and wait for step 0's copies
+    if (tid == 2u * Kw) {
+        for (uint32_t j = 0; j + 2u < RW; ++j) issue_words(j);
+        for (uint32_t j = 0; j + 1u < RP; ++j) issue_pay(j);
+        if (!(landed_words(0) && landed_words(1) && landed_words(2) && landed_words(3) && landed_pay(0))) {
+            latch_error(a.dev, DEV_E_TIMEOUT, 0, tid);
+            s_ab[0] = 1;
+        }
+    }
+    __syncthreads();
+    const bool started = s_ab[0] == 0u;  // false: the prologue gave up a wait, no step runs
+    if (started && !keyw && !prod) {
+        gather(0);
+        gather(1);
+        gather(2);
+        cp_async_wait<2>();
+    }
+    __syncthreads();
+
+    // A thread that gives up a wait in region n raises s_ab[n & 1]; all
+    // threads read it after the barrier of region n, before anyone can write
+    // it again.
+    uint32_t n = 0;
+    bool aborted = !started;
+    for (; started && n <= nst; ++n) {
+        uint32_t odd = 0;
+        if (prod) {
+            if (tid == 2u * Kw) {
+                if (n > 0 && a.decisions) a.decisions[n - 1u] = sel;
+                if (n < nst) {
+                    issue_words(n + RW - 2u);
+                    issue_pay(n + RP - 1u);
+                    if (!(landed_words(n + 4u) && landed_pay(n + 1u))) {
+                        latch_error(a.dev, DEV_E_TIMEOUT, n, tid);
+                        s_ab[n & 1u] = 1;
+                    }
+                }
+            }
+        } else if (keyw) {
+            if (trace && n < nst) trace[n * 8 + 0] = clock64();
+            // every shared load of the step first; then the record warps may
+            // start their copies while this warp hashes
+            uint4 pw[P / 16];
+            uint64_t h = 0;
+            bool hash = false;
+            if (tid < K && n < nst) {
+                const uint32_t m = tid;
+                const uint32_t o = word_of(n, 0)[m];
+                const uint32_t s = word_of(n, 1)[m];
+                const uint32_t l = word_of(n, 2)[m];
+                uint32_t f = kFarSkip;
+                if (s >= a.n_sessions) {
+                    latch_error(a.dev, DEV_E_INDEX, n, m);
+                } else {
+                    const uint32_t x =
+                        unlinked(l, n) ? rec_of(n, m)[0].x : ys[((n - (l >> 16)) % RY) * K + (l & 0xFFFFu)];
+                    uint32_t y = x;
+                    if (x >= a.S || o >= 8u) {
+                        latch_error(a.dev, DEV_E_STATE, n, m);
+                        f = kFarRejected;
+                    } else {
+                        y = tab[sel * a.tab_stride + x * 8u + o];
+                        read_payload_swizzled<P>(pw, pay + static_cast<size_t>(n % RP) * sh.stage_pay, m);
+                        h = h0[x * 8u + o];
+                        hash = true;
+                        f = kFarApplied;
+                    }
+                    ys[(n % RY) * K + m] = y;
+                }
+                fls[(n & 1u) * K + m] = f;
+            }
+            if (trace && n < nst) {
+                asm volatile("" ::"l"(h));
+                trace[n * 8 + 1] = clock64();
+            }
+            named_arrive(1, 2u * Kw);
+            if (hash) {
+                const uint64_t rk = route_key_from<P>(h, pw);
+                rks[(n & 1u) * K + tid] = rk;
+                odd = static_cast<uint32_t>(rk & 1u);
+            }
+            if (trace && n < nst) {
+                asm volatile("" ::"r"(odd));
+                trace[n * 8 + 2] = clock64();
+            }
+        } else {
+            named_sync(1, 2u * Kw);  // the key warps have issued their shared loads
+            gather(n + 3u);
+            if (n >= 1u) record_step(n - 1u, sel_prev);
+            cp_async_wait<2>();  // this thread's copies of step n + 1
+        }
+        // the count of odd keys; the barrier also publishes this region's
+        // states, keys, records and the producer's news
+        const uint32_t total = static_cast<uint32_t>(__syncthreads_count(odd));
+        if (trace && n < nst) trace[n * 8 + 3] = clock64();
+        if (s_ab[n & 1u] != 0u) {
+            aborted = true;
+            break;
+        }
+        if (n < nst) {
+            sel_prev = sel;
+            sel = total > K / 2u ? 1u : 0u;
+        }
+    }
+    // stopped early: the key warps finished step n, the record warps complete it
+    if (started && aborted && n < nst && !keyw && !prod) record_step(n, sel);
+    cp_async_wait<0>();
+    if (tid == 2u * Kw && aborted) {
+        // wait (bounded) for the runs and tiles issued so far
+        const uint32_t w_end = started ? n + RW - 1u : RW - 2u, p_end = started ? n + RP : RP - 1u;
+        for (uint32_t j = n; j < w_end && j < nst; ++j) (void)landed_words(j);
+        for (uint32_t j = n; j < p_end && j < nst; ++j) (void)landed_pay(j);
+    }
+    if (tid == 0 && !aborted) {
         if (nst > 0) a.dev->sel = sel;
         a.dev->step = nst;
     }
@@ -2922,6 +3312,80 @@ cudaError_t launch_link(const StepArgs &a, uint32_t *lnk, cudaStream_t s) {
     const uint32_t threads = a.K >= 512u ? 512u : ((a.K + 31u) / 32u) * 32u;
     k_link<<<grid ? grid : 1u, threads ? threads : 32u, 0, s>>>(a.idx, a.n_sets, a.K, a.n_sessions, lnk);
     return cudaGetLastError();
+}
+
+namespace {
+const void *far_fn(int SB, int P) {
+    return dispatch(SB, P, [](auto b, auto q) {
+        return reinterpret_cast<const void *>(&k_chain_cta_far<decltype(b)::value, decltype(q)::value>);
+    });
+}
+size_t far_smem(const LinkShape &sh, uint32_t K, int SB, uint32_t S, uint32_t tab_stride) {
+    return 1024 + kFarRP * static_cast<size_t>(sh.stage_pay) + kFarRR * static_cast<size_t>(K) * SB +
+           static_cast<size_t>(S) * 64u + 2ull * K * 8u + kFarRW * 3ull * K * 4u + kFarRY * static_cast<size_t>(K) * 4u +
+           2ull * K * 4u + 2ull * tab_stride;
+}
+// Tensor map of the payload rows (P bytes each, n_sets * K rows) in tiles of
+// box_rows rows, swizzled to the row length, as the producer warps load them.
+bool payload_map(const StepArgs &a, int P, uint32_t box_rows, CUtensorMap *map) {
+    EncodeTiled enc = encode_fn();
+    if (!enc) return false;
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(P), static_cast<cuuint64_t>(a.n_sets) * a.K};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(P)};
+    const cuuint32_t box[2] = {static_cast<cuuint32_t>(P), box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUtensorMapSwizzle swz = P == 128 ? CU_TENSOR_MAP_SWIZZLE_128B
+                                   : P == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                             : CU_TENSOR_MAP_SWIZZLE_32B;
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t *>(a.payload), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+}  // namespace
+
+bool chain_cta_far_plan(int SB, int P, uint32_t K, uint32_t S, uint64_t n_sessions, uint32_t tab_stride,
+                        size_t *smem, void *shape_out) {
+    if (K == 0 || K > 256u || K % 8u != 0u || n_sessions > 0xFFFFFFFFull || S == 0 || S > 256u || !encode_fn())
+        return false;
+    LinkShape sh{};
+    sh.prod = 2;
+    sh.n_boxes = 1;
+    sh.box_rows = K;
+    sh.stage_pay = ((K * static_cast<uint32_t>(P)) + 1023u) & ~1023u;
+    const size_t bytes = far_smem(sh, K, SB, S, tab_stride);
+    if (bytes > static_cast<size_t>(max_optin_smem())) return false;
+    *smem = bytes;
+    *static_cast<LinkShape *>(shape_out) = sh;
+    return true;
+}
+
+cudaError_t launch_link_far(const StepArgs &a, uint32_t *lnk, cudaStream_t s) {
+    int dev = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    const uint32_t cap = static_cast<uint32_t>(sms) * 4u;
+    const uint32_t grid = a.n_sets < cap ? a.n_sets : cap;
+    const uint32_t threads = a.K >= 512u ? 512u : ((a.K + 31u) / 32u) * 32u;
+    k_link_far<<<grid ? grid : 1u, threads ? threads : 32u, 0, s>>>(a.idx, a.n_sets, a.K, a.n_sessions, lnk);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_chain_cta_far(const StepArgs &a, int SB, int P, size_t smem, const void *shape,
+                                 const uint32_t *lnk, cudaStream_t s) {
+    const LinkShape &sh = *static_cast<const LinkShape *>(shape);
+    const void *fn = far_fn(SB, P);
+    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    alignas(64) CUtensorMap map;
+    if (!payload_map(a, P, sh.box_rows, &map)) return cudaErrorInvalidValue;
+    StepArgs aa = a;
+    const uint32_t *l = lnk;
+    LinkShape shc = sh;
+    const uint32_t member_threads = ((a.K + 31u) / 32u) * 32u;
+    void *args[] = {&map, &aa, &l, &shc};
+    return cudaLaunchKernel(fn, dim3(1), dim3(2u * member_threads + 32u), args, smem, s);
 }
 
 cudaError_t launch_chain_cta_link(const StepArgs &a, int SB, int P, size_t smem, const void *shape,
