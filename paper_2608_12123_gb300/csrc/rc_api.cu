@@ -91,7 +91,7 @@ struct rc_ctx {
     bool no_pipe = false;   // RC_NO_PIPE=1 selects the plain single-CTA kernel
     bool no_link = false;   // RC_NO_LINK=1 turns off the linked single-CTA kernels
     bool no_prod = false;   // RC_NO_PROD=1 keeps the linked kernel without a producer warp
-    bool use_far = false;   // RC_FAR=1 selects the single-CTA chain with the keys apart from the records
+    bool use_pair = false;  // RC_PAIR=1 selects the single-CTA chain keying two steps per barrier
     bool no_grid_link = false;  // RC_NO_GRID_LINK=1 turns off the grid chain split by links
     bool no_cluster = false;    // RC_NO_CLUSTER=1 turns off the cluster chain (512 < K <= 8192)
     bool use_split = false;  // RC_SPLIT=1 selects the split-phase chain (slower on GB300 so far)
@@ -425,16 +425,16 @@ int run_persist(rc_ctx *c, const rc::StepArgs &a) {
             return RC_OK;
         }
     }
-    if (a.idx && c->use_far && !c->no_pipe && !c->no_link) {
+    if (a.idx && c->use_pair && !c->no_pipe && !c->no_link) {
         size_t smem = 0;
         alignas(8) unsigned char shape[16];
-        if (rc::chain_cta_far_plan(c->SB, c->P, a.K, c->S, c->n_sessions, c->tab_stride, &smem, shape)) {
+        if (rc::chain_cta_pair_plan(c->SB, c->P, a.K, c->S, c->n_sessions, c->tab_stride, &smem, shape)) {
             int rc = ensure(c, c->link_buf, static_cast<size_t>(a.n_sets) * a.K * sizeof(uint32_t));
             if (rc != RC_OK) return rc;
             uint32_t *lnk = static_cast<uint32_t *>(c->link_buf.p);
             c->last_launches = 2;  // link pass + chain
-            RC_CUDA(c, rc::launch_link_far(a, lnk, c->stream));
-            RC_CUDA(c, rc::launch_chain_cta_far(a, c->SB, c->P, smem, shape, lnk, c->stream));
+            RC_CUDA(c, rc::launch_link_pair(a, lnk, c->stream));
+            RC_CUDA(c, rc::launch_chain_cta_pair(a, c->SB, c->P, smem, shape, lnk, c->stream));
             return RC_OK;
         }
     }
@@ -618,8 +618,8 @@ int rc_init(rc_ctx **out, uint32_t S, const uint8_t *table, uint32_t state_bytes
         c->no_link = z && z[0] == '1';
         const char *q = std::getenv("RC_NO_PROD");
         c->no_prod = q && q[0] == '1';
-        const char *fr = std::getenv("RC_FAR");
-        c->use_far = fr && fr[0] == '1';
+        const char *pr = std::getenv("RC_PAIR");
+        c->use_pair = pr && pr[0] == '1';
         const char *gl = std::getenv("RC_NO_GRID_LINK");
         c->no_grid_link = gl && gl[0] == '1';
         const char *cl = std::getenv("RC_NO_CLUSTER");

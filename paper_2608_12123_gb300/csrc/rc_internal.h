@@ -119,15 +119,16 @@ bool chain_cta_link_plan(int state_bytes, int payload_bytes, uint32_t K, uint64_
 cudaError_t launch_link(const StepArgs &a, uint32_t *lnk, cudaStream_t s);
 cudaError_t launch_chain_cta_link(const StepArgs &a, int state_bytes, int payload_bytes, size_t smem,
                                   const void *shape, const uint32_t *lnk, cudaStream_t s);
-// Single-CTA chain with the route keys apart from the records (K <= 256, a
-// multiple of 8): launch_link_far fills lnk (n_sets * K words) with each
-// member's nearest earlier appearance within five cohorts (distance << 16 |
-// position, 0 for none), then the chain runs.  shape_out: 16 bytes.
-bool chain_cta_far_plan(int state_bytes, int payload_bytes, uint32_t K, uint32_t S, uint64_t n_sessions,
-                        uint32_t tab_stride, size_t *smem, void *shape_out);
-cudaError_t launch_link_far(const StepArgs &a, uint32_t *lnk, cudaStream_t s);
-cudaError_t launch_chain_cta_far(const StepArgs &a, int state_bytes, int payload_bytes, size_t smem,
-                                 const void *shape, const uint32_t *lnk, cudaStream_t s);
+// Single-CTA chain keying two steps per block barrier (K <= 256, a multiple
+// of 8, payloads of at most 64 bytes): launch_link_pair fills lnk (n_sets * K
+// words) with each member's nearest earlier appearance within eight cohorts
+// (distance << 16 | position, 0 for none), then the chain runs.  shape_out:
+// 16 bytes.
+bool chain_cta_pair_plan(int state_bytes, int payload_bytes, uint32_t K, uint32_t S, uint64_t n_sessions,
+                         uint32_t tab_stride, size_t *smem, void *shape_out);
+cudaError_t launch_link_pair(const StepArgs &a, uint32_t *lnk, cudaStream_t s);
+cudaError_t launch_chain_cta_pair(const StepArgs &a, int state_bytes, int payload_bytes, size_t smem,
+                                  const void *shape, const uint32_t *lnk, cudaStream_t s);
 cudaError_t chain_grid_size(int state_bytes, int payload_bytes, uint32_t K, int *grid);
 cudaError_t launch_chain_grid(const StepArgs &a, int state_bytes, int payload_bytes, int grid,
                               cudaStream_t s);

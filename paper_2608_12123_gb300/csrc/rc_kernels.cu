@@ -1416,37 +1416,41 @@ __global__ void __launch_bounds__(544, 1)
 }
 
 // ---------------------------------------------------------------------------
-// Links of reach kFarD: for member m of cohort j, the distance t (1..kFarD)
-// to the nearest earlier cohort holding the same session (cohorts taken
-// cyclically, as a chain walks them) and its position q there, packed as
-// t << 16 | q; 0 when none of the kFarD cohorts before holds the session or
-// the index is out of range.  One CTA per cohort, one open-addressing table
-// per earlier cohort (K <= 512 keys in 1,024 slots).
+// Links of reach D: for member m of cohort j, the distance t (1..D) to the
+// nearest earlier cohort holding the same session (cohorts taken cyclically,
+// as a chain walks them) and its position q there, packed as t << 16 | q; 0
+// when none of the D cohorts before holds the session or the index is out of
+// range.  One CTA per cohort, one open-addressing table of SLOTS slots per
+// earlier cohort (at most SLOTS / 2 keys: K <= SLOTS / 2).
 // ---------------------------------------------------------------------------
-constexpr uint32_t kFarD = 5;
+constexpr uint32_t kPairD = 8;  // reach of k_chain_cta_pair's links
 
-__global__ void __launch_bounds__(512) k_link_far(const uint32_t *idx, uint32_t n_sets, uint32_t K, uint64_t N,
-                                                  uint32_t *lnk) {
-    __shared__ uint32_t key[kFarD][kLinkSlots];
-    __shared__ uint16_t pos[kFarD][kLinkSlots];
+template <uint32_t D, uint32_t SLOTS>
+__global__ void __launch_bounds__(512) k_link_reach(const uint32_t *idx, uint32_t n_sets, uint32_t K, uint64_t N,
+                                                    uint32_t *lnk) {
+    static_assert((SLOTS & (SLOTS - 1)) == 0 && SLOTS >= 64 && SLOTS <= 65536, "slots: a power of two");
+    constexpr uint32_t shift = 32u - static_cast<uint32_t>(__builtin_ctz(SLOTS));
+    __shared__ uint32_t key[D][SLOTS];
+    __shared__ uint16_t pos[D][SLOTS];
+    auto hash = [](uint32_t s) { return (s * 0x9E3779B1u) >> shift; };
     for (uint32_t j = blockIdx.x; j < n_sets; j += gridDim.x) {
-        for (uint32_t i = threadIdx.x; i < kFarD * kLinkSlots; i += blockDim.x) (&key[0][0])[i] = kLinkEmpty;
+        for (uint32_t i = threadIdx.x; i < D * SLOTS; i += blockDim.x) (&key[0][0])[i] = kLinkEmpty;
         __syncthreads();
-        for (uint32_t t = 0; t < kFarD; ++t) {
+        for (uint32_t t = 0; t < D; ++t) {
             const uint32_t src =
-                static_cast<uint32_t>((static_cast<uint64_t>(j) + kFarD * static_cast<uint64_t>(n_sets) - 1u - t) %
+                static_cast<uint32_t>((static_cast<uint64_t>(j) + D * static_cast<uint64_t>(n_sets) - 1u - t) %
                                       n_sets);
             for (uint32_t m = threadIdx.x; m < K; m += blockDim.x) {
                 const uint32_t s = __ldg(idx + static_cast<size_t>(src) * K + m);
                 if (s >= N) continue;
-                uint32_t h = link_hash(s);
-                for (uint32_t probe = 0; probe < kLinkSlots; ++probe) {
+                uint32_t h = hash(s);
+                for (uint32_t probe = 0; probe < SLOTS; ++probe) {
                     const uint32_t prev = atomicCAS(&key[t][h], kLinkEmpty, s);
                     if (prev == kLinkEmpty || prev == s) {
                         pos[t][h] = static_cast<uint16_t>(m);
                         break;
                     }
-                    h = (h + 1u) & (kLinkSlots - 1u);
+                    h = (h + 1u) & (SLOTS - 1u);
                 }
             }
         }
@@ -1455,16 +1459,16 @@ __global__ void __launch_bounds__(512) k_link_far(const uint32_t *idx, uint32_t 
             const uint32_t s = __ldg(idx + static_cast<size_t>(j) * K + m);
             uint32_t l = 0;
             if (s < N) {
-                for (uint32_t t = 0; t < kFarD && l == 0u; ++t) {
-                    uint32_t h = link_hash(s);
-                    for (uint32_t probe = 0; probe < kLinkSlots; ++probe) {
+                for (uint32_t t = 0; t < D && l == 0u; ++t) {
+                    uint32_t h = hash(s);
+                    for (uint32_t probe = 0; probe < SLOTS; ++probe) {
                         const uint32_t k = key[t][h];
                         if (k == s) {
                             l = ((t + 1u) << 16) | pos[t][h];
                             break;
                         }
                         if (k == kLinkEmpty) break;
-                        h = (h + 1u) & (kLinkSlots - 1u);
+                        h = (h + 1u) & (SLOTS - 1u);
                     }
                 }
             }
@@ -1474,11 +1478,7 @@ __global__ void __launch_bounds__(512) k_link_far(const uint32_t *idx, uint32_t 
     }
 }
 
-// Named barrier `id` over `count` threads (a multiple of 32): arrive without
-// waiting, or arrive and wait.
-__device__ __forceinline__ void named_arrive(uint32_t id, uint32_t count) {
-    asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(count) : "memory");
-}
+// Named barrier `id` over `count` threads (a multiple of 32): arrive and wait.
 __device__ __forceinline__ void named_sync(uint32_t id, uint32_t count) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
@@ -1497,49 +1497,54 @@ __device__ __forceinline__ uint64_t route_key_from(uint64_t h, const uint4 (&pw)
 
 // ---------------------------------------------------------------------------
 // Persistent chain, one CTA, explicit session indices, K a multiple of 8 up
-// to 256, with the route keys on the decision path and the records off it.
+// to 256, payloads of at most 64 bytes: two steps per block barrier.
 //
-// A key needs the session's state value x (the first word of its record),
-// not the rest of the record.  So x travels on its own: step n leaves, per
-// member, the session's state after the step in a ring Y[n] (the new state,
-// or the old one for a rejected member), and k_link_far gives each member
-// the step (at most kFarD back) and position of its session's previous
-// appearance.  A member of step n takes x from that Y entry or, when its
-// session is not in the kFarD steps before, from its record gathered from
-// HBM three steps ahead.
-//
-// Warps 0 .. ceil(K/32) - 1 (key warps), region n: x; y = T_sel[x][o] into
-// Y[n]; the key from a table of first rounds H0[x][o] and one finaliser
-// round per payload word.  The block barrier then counts the odd keys.
-//
-// The next ceil(K/32) warps (record warps), region n: complete the records
-// of step n - 1 with the keys, new states and decision the key warps left.
-// The input record is the output of the session's previous appearance
-// (record ring, up to kFarD steps back) or the gathered one; the output goes
-// to HBM and to the ring, with the effect.  They also gather, for step n + 3,
-// the records of the members without a link: such a session was last written
-// in step n - 3 or earlier, by region n - 2, which that region's barrier made
-// visible to the CTA.
-//
-// A producer warp streams outcomes, session indices and links (issued six
-// steps ahead) and payload tiles (three ahead), as in k_chain_cta_prod.  The
-// loop runs one region past the last step, in which only the record warps
-// work.  A producer wait that runs out latches RC_E_TIMEOUT; the CTA stops
-// after that region, its record warps first completing the step the key
-// warps finished.  Trace points (thread 0): 0 region start, 1 x ready,
-// 2 key done, 3 after the barrier.
+// The route key of step j depends on the decisions only through the state
+// value x the step reads, and the state a session left in step i is
+// T_{sel_i}[x_i][o_i] with sel_i = d_{i-1}.  So the keys of step j need the
+// decisions up to d_{j-2}, and steps 2r and 2r + 1 can be keyed side by side
+// once d_{2r-1} is known.  Region r (between two block barriers):
+//   key group A (warps 0 .. ceil(K/32) - 1) takes step 2r, key group B (the
+//   next ceil(K/32) warps) step 2r + 1, one member per thread.  x comes from
+//   the session's previous appearance (k_link_reach, up to kPairD steps
+//   back: the input state and outcome that step left in the rings X and O,
+//   and that step's decision) or from its record gathered from HBM.  A
+//   member of step 2r + 1 whose session is in step 2r follows that member's
+//   own link one level further.  The key is a table of first rounds plus one
+//   finaliser round per payload word, the payload read from a swizzled tile.
+//   Two block barriers end the region; their counts are the two groups' odd
+//   keys.
+//   The record group (the next ceil(K/32) warps) completes the records of
+//   steps 2r - 2 and 2r - 1 (a record-group barrier between the two): the
+//   input record is the session's previous output (record ring, up to
+//   kPairD steps back) or the gathered one; the output goes to HBM and to
+//   the ring, with the effect.  It also gathers the records of steps 2r + 4
+//   and 2r + 5 for members without a link: their sessions were last written
+//   in step 2r - 4 or earlier, by region r - 1 at the latest, which that
+//   region's barrier made visible.
+//   The producer lane issues the payload tiles of steps 2r + 2 and 2r + 3,
+//   stores decisions 2r - 2 and 2r - 1, issues the outcome, index and link
+//   runs of steps 2r + 8 and 2r + 9 and waits (bounded) for those runs of
+//   2r + 6 and 2r + 7 and for the two tiles.
+// The loop runs one region past the last key step, in which only the record
+// group works.  A producer wait that runs out latches RC_E_TIMEOUT; the CTA
+// stops after that region, its record group first completing the two steps
+// the key groups finished.  Trace points (thread 0, at step 2r): 0 region
+// start, 1 x ready, 2 key done, 3 after the barrier.
 // ---------------------------------------------------------------------------
-constexpr uint32_t kFarRW = 8;           // word slots (issued six ahead)
-constexpr uint32_t kFarRP = 4;           // payload slots (issued three ahead)
-constexpr uint32_t kFarRR = 10;          // record slots: gather at n - 3 .. last forward at n + 1 + kFarD
-constexpr uint32_t kFarRY = kFarD + 1;   // state-after-step slots
-constexpr uint32_t kFarSkip = 0, kFarRejected = 1, kFarApplied = 2;
+constexpr uint32_t kPairRW = 16;  // word slots
+constexpr uint32_t kPairRR = 16;  // record slots
+constexpr uint32_t kPairRX = 16;  // input-state / outcome slots
+constexpr uint32_t kPairRK = 4;   // key / flag slots
+constexpr uint32_t kPairSkip = 0, kPairRejected = 1, kPairApplied = 2;  // member flags
+constexpr uint32_t kPairRP = 4;   // payload tile slots
 
 template <int SB, int P>
-__global__ void __launch_bounds__(544, 1)
-    k_chain_cta_far(const __grid_constant__ CUtensorMap tmap, StepArgs a, const uint32_t *lnk, LinkShape sh) {
+__global__ void __launch_bounds__(800, 1)
+    k_chain_cta_pair(const __grid_constant__ CUtensorMap tmap, StepArgs a, const uint32_t *lnk, LinkShape sh) {
     constexpr int NV = SB / 16;
-    constexpr uint32_t RW = kFarRW, RP = kFarRP, RR = kFarRR, RY = kFarRY;
+    constexpr int PV = P / 16;
+    constexpr uint32_t RW = kPairRW, RR = kPairRR, RX = kPairRX, RK = kPairRK, RP = kPairRP;
     extern __shared__ uint8_t dsm_raw[];
     __shared__ __align__(8) uint64_t wbar[RW];
     __shared__ __align__(8) uint64_t pbar[RP];
@@ -1547,28 +1552,30 @@ __global__ void __launch_bounds__(544, 1)
     const uint32_t raw = smem_addr(dsm_raw);
     uint8_t *const base = dsm_raw + (((raw + 1023u) & ~1023u) - raw);
     const uint32_t K = a.K;
-    const uint32_t Kw = (K + 31u) & ~31u;  // key threads; record threads next, then the producer warp
+    const uint32_t Kw = (K + 31u) & ~31u;
     const uint32_t tid = threadIdx.x;
-    const bool keyw = tid < Kw;
-    const bool prod = tid >= 2u * Kw;
-    const uint32_t rt = tid - Kw;  // record-thread member (valid when !keyw && !prod)
+    const uint32_t grp = tid / Kw;      // 0: key A, 1: key B, 2: records, 3: producer
+    const uint32_t m = tid - grp * Kw;  // member (groups 0 .. 2)
     const uint32_t nst = a.n_steps;
+    const uint32_t stride = a.tab_stride;
     const uint64_t limit = a.dev->wait_ns;
-    // layout: [payload slots][records][H0][rk][words][Y][flags][tables]
+    // layout: payload tiles [RP] | records [RR][K][NV] | h0 [S][8] | keys [RK][K] |
+    //         words [RW][3][K] | X [RX][K] | O [RX][K] (u8) | flags [RK][K] (u8) | tables
     uint8_t *const pay = base;
-    uint4 *const rec = reinterpret_cast<uint4 *>(base + static_cast<size_t>(RP) * sh.stage_pay);  // [RR][K][NV]
-    uint64_t *const h0 = reinterpret_cast<uint64_t *>(rec + static_cast<size_t>(RR) * K * NV);      // [S][8]
-    uint64_t *const rks = h0 + static_cast<size_t>(a.S) * 8u;                                       // [2][K]
-    uint32_t *const words = reinterpret_cast<uint32_t *>(rks + 2u * K);                           // [RW][3][K]
-    uint32_t *const ys = words + static_cast<size_t>(RW) * 3 * K;                                  // [RY][K]
-    uint32_t *const fls = ys + static_cast<size_t>(RY) * K;                                        // [2][K]
-    uint8_t *const tab = reinterpret_cast<uint8_t *>(fls + 2u * K);
+    uint4 *const rec = reinterpret_cast<uint4 *>(base + static_cast<size_t>(RP) * sh.stage_pay);
+    uint64_t *const h0 = reinterpret_cast<uint64_t *>(rec + static_cast<size_t>(RR) * K * NV);
+    uint64_t *const rks = h0 + static_cast<size_t>(a.S) * 8u;
+    uint32_t *const words = reinterpret_cast<uint32_t *>(rks + static_cast<size_t>(RK) * K);
+    uint32_t *const xs = words + static_cast<size_t>(RW) * 3 * K;
+    uint8_t *const os = reinterpret_cast<uint8_t *>(xs + static_cast<size_t>(RX) * K);
+    uint8_t *const fls = os + static_cast<size_t>(RX) * K;
+    uint8_t *const tab = fls + static_cast<size_t>(RK) * K;
     auto word_of = [&](uint32_t j, uint32_t which) { return words + (static_cast<size_t>(j % RW) * 3 + which) * K; };
-    auto rec_of = [&](uint32_t j, uint32_t m) { return rec + (static_cast<size_t>(j % RR) * K + m) * NV; };
+    auto rec_of = [&](uint32_t j, uint32_t q) { return rec + (static_cast<size_t>(j % RR) * K + q) * NV; };
     const uint64_t stream_pol = policy_evict_first();
     long long *trace = (a.trace && tid == 0) ? a.trace : nullptr;
 
-    // producer lane 0 only
+    // producer lane only
     auto issue_words = [&](uint32_t j) {
         if (j >= nst) return;
         const size_t e0 = static_cast<size_t>(j % a.n_sets) * K;
@@ -1578,58 +1585,120 @@ __global__ void __launch_bounds__(544, 1)
         bulk_load_hint(word_of(j, 1), a.idx + e0, K * 4u, b, stream_pol);
         bulk_load_hint(word_of(j, 2), lnk + e0, K * 4u, b, stream_pol);
     };
+    auto landed_words = [&](uint32_t j) { return j >= nst || mbar_wait_bounded(&wbar[j % RW], (j / RW) & 1u, limit); };
     auto issue_pay = [&](uint32_t j) {
         if (j >= nst) return;
         const uint32_t st = j % RP;
-        const int32_t row0 = static_cast<int32_t>((j % a.n_sets) * K);
-        mbar_arrive_expect_tx(&pbar[st], sh.n_boxes * sh.box_rows * P);
-        for (uint32_t b = 0; b < sh.n_boxes; ++b)
-            tma_load_2d_hint(pay + static_cast<size_t>(st) * sh.stage_pay + b * sh.box_rows * P, &tmap, 0,
-                             row0 + static_cast<int32_t>(b * sh.box_rows), &pbar[st], stream_pol);
+        mbar_arrive_expect_tx(&pbar[st], sh.box_rows * P);
+        tma_load_2d_hint(pay + static_cast<size_t>(st) * sh.stage_pay, &tmap, 0,
+                         static_cast<int32_t>((j % a.n_sets) * K), &pbar[st], stream_pol);
     };
-    auto landed_words = [&](uint32_t j) { return j >= nst || mbar_wait_bounded(&wbar[j % RW], (j / RW) & 1u, limit); };
     auto landed_pay = [&](uint32_t j) { return j >= nst || mbar_wait_bounded(&pbar[j % RP], (j / RP) & 1u, limit); };
-    // a member of step j without a usable link: its record comes from HBM
     auto unlinked = [](uint32_t l, uint32_t j) {
         const uint32_t t = l >> 16;
         return t == 0u || t > j;
     };
-    // record thread: gather its member's record of step j when unlinked (one
-    // commit group, empty when there is nothing to copy)
+
+    const uint32_t sel0 = ld_volatile_u32(&a.dev->sel) & 1u;
+    uint64_t dv = 0;  // bit (i & 63): decision d_i, for the steps decided so far
+    auto sel_of = [&](uint32_t j) -> uint32_t {
+        return j == 0u ? sel0 : static_cast<uint32_t>((dv >> ((j - 1u) & 63u)) & 1u);
+    };
+    // the state member q of step j left its session in (rings X and O of step j)
+    auto after = [&](uint32_t j, uint32_t q) -> uint32_t {
+        const uint32_t x = xs[(j % RX) * K + q];
+        const uint32_t o = os[(j % RX) * K + q];
+        return (x < a.S && o < 8u) ? static_cast<uint32_t>(tab[sel_of(j) * stride + x * 8u + o]) : x;
+    };
+
+    // key thread: the outcome, index and link of its next step, loaded a
+    // region ahead
+    auto key_prefetch = [&](uint32_t j, uint32_t &o, uint32_t &s, uint32_t &l) {
+        if (j < nst && m < K) {
+            o = word_of(j, 0)[m];
+            s = word_of(j, 1)[m];
+            l = word_of(j, 2)[m];
+        }
+    };
+    // key thread: x, the rings X and O, the key and the flag of its member of
+    // step j; `chase` for group B (a session in step j - 1 is in this region)
+    auto key_step = [&](uint32_t j, bool chase, uint32_t o, uint32_t s, uint32_t l) {
+        uint32_t odd = 0;
+        if (j >= nst || m >= K) return odd;
+        uint4 pw[PV];
+        read_payload_swizzled<P>(pw, pay + static_cast<size_t>(j % RP) * sh.stage_pay, m);
+        uint32_t f = kPairSkip;
+        if (s >= a.n_sessions) {
+            latch_error(a.dev, DEV_E_INDEX, j, m);
+        } else {
+            const uint32_t t = l >> 16, q = l & 0xFFFFu;
+            uint32_t x;
+            if (t == 0u || t > j) {
+                x = rec_of(j, m)[0].x;
+            } else if (chase && t == 1u) {
+                const uint32_t i = j - 1u;
+                const uint32_t l2 = word_of(i, 2)[q];
+                const uint32_t oi = word_of(i, 0)[q];
+                const uint32_t xi = unlinked(l2, i) ? rec_of(i, q)[0].x : after(i - (l2 >> 16), l2 & 0xFFFFu);
+                x = (xi < a.S && oi < 8u) ? static_cast<uint32_t>(tab[sel_of(i) * stride + xi * 8u + oi]) : xi;
+            } else {
+                x = after(j - t, q);
+            }
+            if (trace) {
+                asm volatile("" ::"r"(x));
+                trace[j * 8 + 1] = clock64();
+            }
+            xs[(j % RX) * K + m] = x;
+            os[(j % RX) * K + m] = static_cast<uint8_t>(o < 8u ? o : 8u);
+            if (x >= a.S || o >= 8u) {
+                latch_error(a.dev, DEV_E_STATE, j, m);
+                f = kPairRejected;
+            } else {
+                const uint64_t rk = route_key_from<P>(h0[x * 8u + o], pw);
+                rks[(j % RK) * K + m] = rk;
+                odd = static_cast<uint32_t>(rk & 1u);
+                f = kPairApplied;
+            }
+        }
+        fls[(j % RK) * K + m] = static_cast<uint8_t>(f);
+        return odd;
+    };
+    // record thread: gather its member's record of step j when it has no link
     auto gather = [&](uint32_t j) {
-        if (j < nst && rt < K) {
-            const uint32_t s = word_of(j, 1)[rt];
-            if (s < a.n_sessions && unlinked(word_of(j, 2)[rt], j)) {
+        if (j < nst && m < K) {
+            const uint32_t s = word_of(j, 1)[m];
+            if (s < a.n_sessions && unlinked(word_of(j, 2)[m], j)) {
                 const uint4 *rp = reinterpret_cast<const uint4 *>(a.state + static_cast<size_t>(s) * SB);
-                uint4 *dst = rec_of(j, rt);
+                uint4 *dst = rec_of(j, m);
 #pragma unroll
                 for (int k = 0; k < NV; ++k) cp_async16(dst + k, rp + k);
             }
         }
-        cp_async_commit();
     };
-    // record thread: complete its member's record of step j (decision sel_j)
-    auto record_step = [&](uint32_t j, uint32_t sel_j) {
-        if (rt >= K) return;
-        const uint32_t f = fls[(j & 1u) * K + rt];
-        if (f == kFarSkip) return;
-        const uint32_t l = word_of(j, 2)[rt];
-        uint4 *mine = rec_of(j, rt);
+    // record thread: complete its member's record of step j
+    auto record_step = [&](uint32_t j) {
+        if (j >= nst || m >= K) return;
+        const uint32_t f = fls[(j % RK) * K + m];
+        if (f == kPairSkip) return;
+        const uint32_t l = word_of(j, 2)[m];
+        uint4 *mine = rec_of(j, m);
         const uint4 *src = unlinked(l, j) ? mine : rec_of(j - (l >> 16), l & 0xFFFFu);
         uint4 r[NV];
 #pragma unroll
         for (int k = 0; k < NV; ++k) r[k] = src[k];
-        if (f == kFarRejected) {
+        if (f == kPairRejected) {
             if (src != mine) {
 #pragma unroll
                 for (int k = 0; k < NV; ++k) mine[k] = r[k];
             }
             return;
         }
-        const uint32_t o = word_of(j, 0)[rt];
-        const uint32_t s = word_of(j, 1)[rt];
-        const uint32_t y = ys[(j % RY) * K + rt];
-        const uint64_t rk = rks[(j & 1u) * K + rt];
+        const uint32_t o = word_of(j, 0)[m];
+        const uint32_t s = word_of(j, 1)[m];
+        const uint32_t x = xs[(j % RX) * K + m];
+        const uint32_t sel = sel_of(j);
+        const uint32_t y = tab[sel * stride + x * 8u + o];
+        const uint64_t rk = rks[(j % RK) * K + m];
         r[0].x = y;
         r[0].y = r[0].y + 1u;
         mix_acc<SB>(r, rk);
@@ -1639,13 +1708,13 @@ __global__ void __launch_bounds__(544, 1)
             mine[k] = r[k];
             rp[k] = r[k];
         }
-        const size_t slot = static_cast<size_t>(j) * K + rt;
+        const size_t slot = static_cast<size_t>(j) * K + m;
         if (a.effects) {
             uint4 e;
             e.x = static_cast<uint32_t>(rk);
             e.y = static_cast<uint32_t>(rk >> 32);
             e.z = s;
-            e.w = y | (o << 16) | (sel_j << 24);
+            e.w = y | (o << 16) | (sel << 24);
             __stcs(reinterpret_cast<uint4 *>(a.effects) + slot, e);
         }
         if (a.state_log) {
@@ -1662,128 +1731,130 @@ __global__ void __launch_bounds__(544, 1)
         s_ab[0] = 0;
         s_ab[1] = 0;
     }
-    stage_tables(tab, a.tables, a.tab_stride, 2, 0);
+    stage_tables(tab, a.tables, stride, 2, 0);
     for (uint32_t i = tid; i < a.S * 8u; i += blockDim.x) h0[i] = fin64(pack64(i >> 3, i & 7u) ^ kGamma);
-    uint32_t sel = ld_volatile_u32(&a.dev->sel) & 1u;
-    uint32_t sel_prev = sel;
     __syncthreads();
-    // prologue: runs of steps 0..6 and tiles of steps 0..2 go out; the runs
-    // of steps 0..3 and the tiles of step 0 are waited for; the record warps
-    // then gather steps 0, 1 and 2 and wait for step 0's copies
-    if (tid == 2u * Kw) {
-        for (uint32_t j = 0; j + 2u < RW; ++j) issue_words(j);
-        for (uint32_t j = 0; j + 1u < RP; ++j) issue_pay(j);
-        if (!(landed_words(0) && landed_words(1) && landed_words(2) && landed_words(3) && landed_pay(0))) {
+    // prologue: runs of steps 0..7 and tiles of steps 0 and 1 go out; the
+    // runs of 0..5 and the tiles are waited for; then the record group gathers
+    // steps 0..3 (two copy groups) and waits for the first, and the key groups
+    // load their steps 0 and 1
+    const uint32_t prod_lane = 3u * Kw;
+    if (tid == prod_lane) {
+        for (uint32_t j = 0; j < 8u; ++j) issue_words(j);
+        issue_pay(0);
+        issue_pay(1);
+        bool ok = landed_pay(0) && landed_pay(1);
+        for (uint32_t j = 0; j < 6u; ++j) ok = ok && landed_words(j);
+        if (!ok) {
             latch_error(a.dev, DEV_E_TIMEOUT, 0, tid);
             s_ab[0] = 1;
         }
     }
     __syncthreads();
     const bool started = s_ab[0] == 0u;  // false: the prologue gave up a wait, no step runs
-    if (started && !keyw && !prod) {
-        gather(0);
-        gather(1);
-        gather(2);
-        cp_async_wait<2>();
+    uint32_t o_a = 0, s_a = 0, l_a = 0, o_b = 0, s_b = 0, l_b = 0;
+    if (started) {
+        if (grp == 2u) {
+            gather(0);
+            gather(1);
+            cp_async_commit();
+            gather(2);
+            gather(3);
+            cp_async_commit();
+            cp_async_wait<1>();
+        } else if (grp < 2u) {
+            key_prefetch(grp, o_a, s_a, l_a);
+        }
     }
     __syncthreads();
 
-    // A thread that gives up a wait in region n raises s_ab[n & 1]; all
-    // threads read it after the barrier of region n, before anyone can write
-    // it again.
-    uint32_t n = 0;
+    // the last region: its key steps are past the end, the record group
+    // completes the last two steps
+    const uint32_t r_end = nst == 0u ? 0u : (nst - 1u) / 2u + 1u;
+    uint32_t r = 0;
     bool aborted = !started;
-    for (; started && n <= nst; ++n) {
-        uint32_t odd = 0;
-        if (prod) {
-            if (tid == 2u * Kw) {
-                if (n > 0 && a.decisions) a.decisions[n - 1u] = sel;
-                if (n < nst) {
-                    issue_words(n + RW - 2u);
-                    issue_pay(n + RP - 1u);
-                    if (!(landed_words(n + 4u) && landed_pay(n + 1u))) {
-                        latch_error(a.dev, DEV_E_TIMEOUT, n, tid);
-                        s_ab[n & 1u] = 1;
-                    }
+    for (; started && r <= r_end; ++r) {
+        const uint32_t ja = 2u * r, jb = ja + 1u;
+        uint32_t odd_a = 0, odd_b = 0;
+        if (grp == 3u) {
+            if (tid == prod_lane) {
+                issue_pay(ja + 2u);
+                issue_pay(ja + 3u);
+                if (a.decisions && r > 0) {
+                    if (ja - 2u < nst) a.decisions[ja - 2u] = sel_of(ja - 1u);
+                    if (ja - 1u < nst) a.decisions[ja - 1u] = sel_of(ja);
+                }
+                issue_words(ja + 8u);
+                issue_words(ja + 9u);
+                if (!(landed_words(ja + 6u) && landed_words(ja + 7u) && landed_pay(ja + 2u) &&
+                      landed_pay(ja + 3u))) {
+                    latch_error(a.dev, DEV_E_TIMEOUT, ja, tid);
+                    s_ab[r & 1u] = 1;
                 }
             }
-        } else if (keyw) {
-            if (trace && n < nst) trace[n * 8 + 0] = clock64();
-            // every shared load of the step first; then the record warps may
-            // start their copies while this warp hashes
-            uint4 pw[P / 16];
-            uint64_t h = 0;
-            bool hash = false;
-            if (tid < K && n < nst) {
-                const uint32_t m = tid;
-                const uint32_t o = word_of(n, 0)[m];
-                const uint32_t s = word_of(n, 1)[m];
-                const uint32_t l = word_of(n, 2)[m];
-                uint32_t f = kFarSkip;
-                if (s >= a.n_sessions) {
-                    latch_error(a.dev, DEV_E_INDEX, n, m);
-                } else {
-                    const uint32_t x =
-                        unlinked(l, n) ? rec_of(n, m)[0].x : ys[((n - (l >> 16)) % RY) * K + (l & 0xFFFFu)];
-                    uint32_t y = x;
-                    if (x >= a.S || o >= 8u) {
-                        latch_error(a.dev, DEV_E_STATE, n, m);
-                        f = kFarRejected;
-                    } else {
-                        y = tab[sel * a.tab_stride + x * 8u + o];
-                        read_payload_swizzled<P>(pw, pay + static_cast<size_t>(n % RP) * sh.stage_pay, m);
-                        h = h0[x * 8u + o];
-                        hash = true;
-                        f = kFarApplied;
-                    }
-                    ys[(n % RY) * K + m] = y;
-                }
-                fls[(n & 1u) * K + m] = f;
-            }
-            if (trace && n < nst) {
-                asm volatile("" ::"l"(h));
-                trace[n * 8 + 1] = clock64();
-            }
-            named_arrive(1, 2u * Kw);
-            if (hash) {
-                const uint64_t rk = route_key_from<P>(h, pw);
-                rks[(n & 1u) * K + tid] = rk;
-                odd = static_cast<uint32_t>(rk & 1u);
-            }
-            if (trace && n < nst) {
+        } else if (grp < 2u) {
+            const uint32_t j = ja + grp;
+            if (trace && j < nst) trace[j * 8 + 0] = clock64();
+            // this step's inputs are in (o_a, s_a, l_a); the next step's go to
+            // the b set, and the roles swap below
+            key_prefetch(j + 2u, o_b, s_b, l_b);
+            const uint32_t odd = key_step(j, grp == 1u, o_a, s_a, l_a);
+            if (grp == 0u)
+                odd_a = odd;
+            else
+                odd_b = odd;
+            if (trace && j < nst) {
                 asm volatile("" ::"r"(odd));
-                trace[n * 8 + 2] = clock64();
+                trace[j * 8 + 2] = clock64();
             }
-        } else {
-            named_sync(1, 2u * Kw);  // the key warps have issued their shared loads
-            gather(n + 3u);
-            if (n >= 1u) record_step(n - 1u, sel_prev);
-            cp_async_wait<2>();  // this thread's copies of step n + 1
+            o_a = o_b;
+            s_a = s_b;
+            l_a = l_b;
+        } else if (grp == 2u) {
+            gather(ja + 4u);
+            gather(ja + 5u);
+            cp_async_commit();
+            if (r > 0) record_step(ja - 2u);
+            named_sync(2, Kw);
+            if (r > 0) record_step(ja - 1u);
+            cp_async_wait<1>();  // this thread's copies of steps 2r + 2 and 2r + 3
         }
-        // the count of odd keys; the barrier also publishes this region's
-        // states, keys, records and the producer's news
-        const uint32_t total = static_cast<uint32_t>(__syncthreads_count(odd));
-        if (trace && n < nst) trace[n * 8 + 3] = clock64();
-        if (s_ab[n & 1u] != 0u) {
+        // the counts of the two groups' odd keys, one block barrier each; the
+        // first also publishes this region's rings, records and the
+        // producer's news
+        const uint32_t total_a = static_cast<uint32_t>(__syncthreads_count(odd_a));
+        const uint32_t total_b = static_cast<uint32_t>(__syncthreads_count(odd_b));
+        if (trace && ja < nst) trace[ja * 8 + 3] = clock64();
+        if (ja < nst) {
+            const uint32_t da = total_a > K / 2u ? 1u : 0u;
+            dv = (dv & ~(1ull << (ja & 63u))) | (static_cast<uint64_t>(da) << (ja & 63u));
+        }
+        if (jb < nst) {
+            const uint32_t db = total_b > K / 2u ? 1u : 0u;
+            dv = (dv & ~(1ull << (jb & 63u))) | (static_cast<uint64_t>(db) << (jb & 63u));
+        }
+        if (s_ab[r & 1u] != 0u) {
             aborted = true;
             break;
         }
-        if (n < nst) {
-            sel_prev = sel;
-            sel = total > K / 2u ? 1u : 0u;
-        }
     }
-    // stopped early: the key warps finished step n, the record warps complete it
-    if (started && aborted && n < nst && !keyw && !prod) record_step(n, sel);
+    // stopped early: the key groups finished steps 2r and 2r + 1, the record
+    // group completes them
+    if (started && aborted && grp == 2u) {
+        record_step(2u * r);
+        named_sync(2, Kw);
+        record_step(2u * r + 1u);
+    }
     cp_async_wait<0>();
-    if (tid == 2u * Kw && aborted) {
-        // wait (bounded) for the runs and tiles issued so far
-        const uint32_t w_end = started ? n + RW - 1u : RW - 2u, p_end = started ? n + RP : RP - 1u;
-        for (uint32_t j = n; j < w_end && j < nst; ++j) (void)landed_words(j);
-        for (uint32_t j = n; j < p_end && j < nst; ++j) (void)landed_pay(j);
+    if (tid == prod_lane && aborted) {
+        // wait (bounded) for the runs and tiles still in flight
+        const uint32_t j0 = started ? 2u * r + 6u : 0u, j1 = started ? 2u * r + 10u : 8u;
+        for (uint32_t j = j0; j < j1 && j < nst; ++j) (void)landed_words(j);
+        const uint32_t p0 = started ? 2u * r + 2u : 0u, p1 = p0 + 2u;
+        for (uint32_t j = p0; j < p1 && j < nst; ++j) (void)landed_pay(j);
     }
     if (tid == 0 && !aborted) {
-        if (nst > 0) a.dev->sel = sel;
+        if (nst > 0) a.dev->sel = sel_of(nst);
         a.dev->step = nst;
     }
 }
@@ -3315,16 +3386,6 @@ cudaError_t launch_link(const StepArgs &a, uint32_t *lnk, cudaStream_t s) {
 }
 
 namespace {
-const void *far_fn(int SB, int P) {
-    return dispatch(SB, P, [](auto b, auto q) {
-        return reinterpret_cast<const void *>(&k_chain_cta_far<decltype(b)::value, decltype(q)::value>);
-    });
-}
-size_t far_smem(const LinkShape &sh, uint32_t K, int SB, uint32_t S, uint32_t tab_stride) {
-    return 1024 + kFarRP * static_cast<size_t>(sh.stage_pay) + kFarRR * static_cast<size_t>(K) * SB +
-           static_cast<size_t>(S) * 64u + 2ull * K * 8u + kFarRW * 3ull * K * 4u + kFarRY * static_cast<size_t>(K) * 4u +
-           2ull * K * 4u + 2ull * tab_stride;
-}
 // Tensor map of the payload rows (P bytes each, n_sets * K rows) in tiles of
 // box_rows rows, swizzled to the row length, as the producer warps load them.
 bool payload_map(const StepArgs &a, int P, uint32_t box_rows, CUtensorMap *map) {
@@ -3343,39 +3404,58 @@ bool payload_map(const StepArgs &a, int P, uint32_t box_rows, CUtensorMap *map) 
 }
 }  // namespace
 
-bool chain_cta_far_plan(int SB, int P, uint32_t K, uint32_t S, uint64_t n_sessions, uint32_t tab_stride,
-                        size_t *smem, void *shape_out) {
-    if (K == 0 || K > 256u || K % 8u != 0u || n_sessions > 0xFFFFFFFFull || S == 0 || S > 256u || !encode_fn())
+namespace {
+const void *pair_fn(int SB, int P) {
+    return dispatch(SB, P, [](auto b, auto q) -> const void * {
+        constexpr int B = decltype(b)::value, Q = decltype(q)::value;
+        if constexpr (Q <= 64) return reinterpret_cast<const void *>(&k_chain_cta_pair<B, Q>);
+        return nullptr;
+    });
+}
+size_t pair_smem(uint32_t K, int SB, uint32_t S, uint32_t tab_stride, uint32_t stage_pay) {
+    return 1024 + kPairRP * static_cast<size_t>(stage_pay) + kPairRR * static_cast<size_t>(K) * SB + static_cast<size_t>(S) * 64u + kPairRK * 8ull * K +
+           kPairRW * 12ull * K + kPairRX * 4ull * K + kPairRX * static_cast<size_t>(K) + kPairRK * static_cast<size_t>(K) +
+           2ull * tab_stride;
+}
+}  // namespace
+
+bool chain_cta_pair_plan(int SB, int P, uint32_t K, uint32_t S, uint64_t n_sessions, uint32_t tab_stride,
+                         size_t *smem, void *shape_out) {
+    if (K == 0 || K > 256u || K % 8u != 0u || P > 64 || n_sessions > 0xFFFFFFFFull || S == 0 || S > 256u ||
+        !encode_fn())
         return false;
     LinkShape sh{};
-    sh.prod = 2;
+    sh.prod = 3;
     sh.n_boxes = 1;
     sh.box_rows = K;
     sh.stage_pay = ((K * static_cast<uint32_t>(P)) + 1023u) & ~1023u;
-    const size_t bytes = far_smem(sh, K, SB, S, tab_stride);
+    const size_t bytes = pair_smem(K, SB, S, tab_stride, sh.stage_pay);
     if (bytes > static_cast<size_t>(max_optin_smem())) return false;
     *smem = bytes;
     *static_cast<LinkShape *>(shape_out) = sh;
     return true;
 }
 
-cudaError_t launch_link_far(const StepArgs &a, uint32_t *lnk, cudaStream_t s) {
+cudaError_t launch_link_pair(const StepArgs &a, uint32_t *lnk, cudaStream_t s) {
     int dev = 0, sms = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return e;
+    if (a.K > 256u) return cudaErrorInvalidValue;  // the tables hold 512 slots
     const uint32_t cap = static_cast<uint32_t>(sms) * 4u;
     const uint32_t grid = a.n_sets < cap ? a.n_sets : cap;
-    const uint32_t threads = a.K >= 512u ? 512u : ((a.K + 31u) / 32u) * 32u;
-    k_link_far<<<grid ? grid : 1u, threads ? threads : 32u, 0, s>>>(a.idx, a.n_sets, a.K, a.n_sessions, lnk);
+    const uint32_t threads = ((a.K + 31u) / 32u) * 32u;
+    k_link_reach<kPairD, 512><<<grid ? grid : 1u, threads ? threads : 32u, 0, s>>>(a.idx, a.n_sets, a.K,
+                                                                                   a.n_sessions, lnk);
     return cudaGetLastError();
 }
 
-cudaError_t launch_chain_cta_far(const StepArgs &a, int SB, int P, size_t smem, const void *shape,
-                                 const uint32_t *lnk, cudaStream_t s) {
+cudaError_t launch_chain_cta_pair(const StepArgs &a, int SB, int P, size_t smem, const void *shape,
+                                  const uint32_t *lnk, cudaStream_t s) {
     const LinkShape &sh = *static_cast<const LinkShape *>(shape);
-    const void *fn = far_fn(SB, P);
+    const void *fn = pair_fn(SB, P);
+    if (!fn) return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     alignas(64) CUtensorMap map;
@@ -3383,9 +3463,9 @@ cudaError_t launch_chain_cta_far(const StepArgs &a, int SB, int P, size_t smem, 
     StepArgs aa = a;
     const uint32_t *l = lnk;
     LinkShape shc = sh;
-    const uint32_t member_threads = ((a.K + 31u) / 32u) * 32u;
     void *args[] = {&map, &aa, &l, &shc};
-    return cudaLaunchKernel(fn, dim3(1), dim3(2u * member_threads + 32u), args, smem, s);
+    const uint32_t member_threads = ((a.K + 31u) / 32u) * 32u;
+    return cudaLaunchKernel(fn, dim3(1), dim3(3u * member_threads + 32u), args, smem, s);
 }
 
 cudaError_t launch_chain_cta_link(const StepArgs &a, int SB, int P, size_t smem, const void *shape,

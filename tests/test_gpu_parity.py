@@ -227,19 +227,19 @@ def test_grid_barrier_wait_is_bounded_every_grid_kernel(g, rc, monkeypatch, kern
         rc.rc_free(ctx)
 
 
-@pytest.mark.parametrize("kernel", ["owned", "split", "far", "prod", "link", "plain"])
+@pytest.mark.parametrize("kernel", ["owned", "split", "pair", "prod", "link", "plain"])
 @pytest.mark.parametrize("P", [32, 64, 128])
 @pytest.mark.parametrize("K,N", [(8, 9), (64, 67), (64, 128), (256, 259), (256, 512), (256, 1500), (496, 1000),
                                  (512, 513), (100, 300), (256, 1 << 20)])
 def test_small_cohort_repeated_sessions(g, rc, monkeypatch, kernel, P, K, N):
     """Sessions that recur in consecutive steps at other member positions: each
-    persistent kernel must see the records the previous step wrote ("far": the
-    single-CTA chain with the keys apart from the records, K <= 256)."""
+    persistent kernel must see the records the previous step wrote ("pair":
+    the single-CTA chain keying two steps per barrier, K <= 256 and P <= 64)."""
     monkeypatch.setenv("RC_OWNED", "1" if kernel == "owned" else "0")
     monkeypatch.setenv("RC_SPLIT", "1" if kernel == "split" else "0")
     monkeypatch.setenv("RC_NO_PIPE", "1" if kernel == "plain" else "0")
     monkeypatch.setenv("RC_NO_PROD", "1" if kernel == "link" else "0")
-    monkeypatch.setenv("RC_FAR", "1" if kernel == "far" else "0")
+    monkeypatch.setenv("RC_PAIR", "1" if kernel == "pair" else "0")
     tables, state0, outc, pay, idx = _inputs(60 + K % 13 + P, K, 64, 16, P, 40, N=N)
     n = 40
     want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=1)
@@ -259,26 +259,27 @@ def test_single_cta_identity_sessions(g, rc, monkeypatch, pipe, SB, P, K):
     g.assert_same(got, want, f"identity pipe={pipe} SB={SB} P={P} K={K}")
 
 
-@pytest.mark.parametrize("far", [True, False])
+@pytest.mark.parametrize("kernel", ["pair", "prod"])
 @pytest.mark.parametrize("n_sets", [1, 2, 3, 7])
 @pytest.mark.parametrize("SB,P,K,extra,want_launches", [(16, 64, 256, 0, 2), (16, 64, 256, 1, 2), (16, 32, 7, 2, 2),
                                                    (64, 64, 256, 1, 2), (16, 128, 300, 3, 2), (64, 32, 33, 0, 2),
                                                    (16, 64, 264, 9, 2), (16, 64, 512, 5, 2), (64, 128, 512, 1, 1),
                                                    (64, 128, 64, 3, 2), (16, 32, 8, 0, 2), (16, 128, 248, 40, 2)])
-def test_linked_single_cta_ring_wraps(g, rc, monkeypatch, SB, P, K, extra, want_launches, n_sets, far):
+def test_linked_single_cta_ring_wraps(g, rc, monkeypatch, SB, P, K, extra, want_launches, n_sets, kernel):
     """The single-CTA chains that take recurring sessions from shared rings:
     cohorts drawn from N = K + extra sessions, so nearly every session recurs
     in the next steps at another position, and a ring of 1, 2, 3 or 7 cohorts,
-    so links wrap (with one cohort every member follows itself).  With far, K
-    a multiple of 8 up to 256 takes the chain with the keys apart from the
-    records where its rings fit (links five cohorts back); otherwise K a
+    so links wrap (with one cohort every member follows itself).  K a
+    multiple of 8 up to 256 takes, where its rings fit, the selected chain:
+    "pair" (two steps per barrier, links eight cohorts back, P <= 64) or
+    "prod"; otherwise K a
     multiple of 8 takes the producer-warp form (payload tiles: one, or two for
     K > 256), other K the per-thread-copy form.  Both launches (link pass and
     chain) are counted where the kernel applies; 512 members with 64-byte
     records and 128-byte payloads do not fit its rings and take the plain
     single-CTA kernel (one launch)."""
     import torch
-    monkeypatch.setenv("RC_FAR", "1" if far else "0")
+    monkeypatch.setenv("RC_PAIR", "1" if kernel == "pair" else "0")
     S = 256 if SB == 64 else 64
     N = K + extra
     tables, state0, outc, pay, idx = _inputs(90 + n_sets + K % 7, K, S, SB, P, n_sets, N=N)
