@@ -12,6 +12,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <string>
+#include <algorithm>
 #include <vector>
 
 #include "rc.h"
@@ -85,6 +86,9 @@ struct rc_ctx {
     CachedGraph cond, floor;
     NestedGraphs nested;
     cudaEvent_t ev_start = nullptr, ev_stop = nullptr;
+    cudaStream_t copy_stream = nullptr;  // host -> device copies of a chain run in pieces
+    cudaStream_t out_stream = nullptr;   // device -> host copies of a chain run in pieces
+    std::vector<cudaEvent_t> pipe_ev;    // per piece: inputs copied, piece done
     double last_ms = 0.0;
     uint32_t last_launches = 0;
     bool no_tma = false;   // RC_NO_TMA=1 in the environment selects the plain grid kernel
@@ -92,6 +96,7 @@ struct rc_ctx {
     bool no_link = false;   // RC_NO_LINK=1 turns off the linked single-CTA kernels
     bool no_prod = false;   // RC_NO_PROD=1 keeps the linked kernel without a producer warp
     bool use_pair = false;  // RC_PAIR=1 selects the single-CTA chain keying two steps per barrier
+    bool no_pieces = false; // RC_NO_PIECES=1 stages host-memory events whole (no pieces)
     bool no_grid_link = false;  // RC_NO_GRID_LINK=1 turns off the grid chain split by links
     bool no_cluster = false;    // RC_NO_CLUSTER=1 turns off the cluster chain (512 < K <= 8192)
     bool use_split = false;  // RC_SPLIT=1 selects the split-phase chain (slower on GB300 so far)
@@ -196,8 +201,10 @@ int finish(rc_ctx *c) {
 struct Resolved {
     rc::StepArgs a{};
     bool host_dec = false, host_eff = false, host_log = false;
+    bool host_out = false, host_pay = false, host_idx = false;  // inputs not yet copied (defer_inputs)
     uint32_t *user_dec = nullptr;
     void *user_eff = nullptr, *user_log = nullptr;
+    const rc_events *user_ev = nullptr;
 };
 
 int check_events(rc_ctx *c, const rc_events *ev, uint32_t K) {
@@ -212,9 +219,10 @@ int check_events(rc_ctx *c, const rc_events *ev, uint32_t K) {
 }
 
 // Fills the kernel arguments; event and output buffers in host memory are
-// staged through device buffers (inputs copied now, outputs after the work).
+// staged through device buffers (inputs copied now, or by the caller when
+// defer_inputs; outputs after the work).
 int resolve(rc_ctx *c, void *state, const rc_events *ev, uint32_t K, uint32_t n_steps, uint32_t *dec,
-            void *eff, void *slog, bool dec_is_input, Resolved *r) {
+            void *eff, void *slog, bool dec_is_input, Resolved *r, bool defer_inputs = false) {
     int rc = check_events(c, ev, K);
     if (rc != RC_OK) return rc;
     if (!state || !aligned16(state)) return fail(c, RC_E_INVAL, "state must be a 16-byte aligned device pointer");
@@ -238,22 +246,31 @@ int resolve(rc_ctx *c, void *state, const rc_events *ev, uint32_t K, uint32_t n_
     a.outcome = ev->outcome;
     a.payload = ev->payload;
     a.idx = ev->session_idx;
+    r->user_ev = ev;
     if (K > 0) {
         if (is_host_ptr(ev->outcome)) {
             if ((rc = ensure(c, c->st_outcome, n_ev * 4)) != RC_OK) return rc;
-            RC_CUDA(c, cudaMemcpyAsync(c->st_outcome.p, ev->outcome, n_ev * 4, cudaMemcpyHostToDevice, c->stream));
+            if (!defer_inputs)
+                RC_CUDA(c, cudaMemcpyAsync(c->st_outcome.p, ev->outcome, n_ev * 4, cudaMemcpyHostToDevice,
+                                           c->stream));
             a.outcome = static_cast<const uint32_t *>(c->st_outcome.p);
+            r->host_out = defer_inputs;
         }
         if (is_host_ptr(ev->payload)) {
             if ((rc = ensure(c, c->st_payload, n_ev * c->P)) != RC_OK) return rc;
-            RC_CUDA(c, cudaMemcpyAsync(c->st_payload.p, ev->payload, n_ev * c->P, cudaMemcpyHostToDevice,
-                                       c->stream));
+            if (!defer_inputs)
+                RC_CUDA(c, cudaMemcpyAsync(c->st_payload.p, ev->payload, n_ev * c->P, cudaMemcpyHostToDevice,
+                                           c->stream));
             a.payload = static_cast<const uint8_t *>(c->st_payload.p);
+            r->host_pay = defer_inputs;
         }
         if (ev->session_idx && is_host_ptr(ev->session_idx)) {
             if ((rc = ensure(c, c->st_idx, n_ev * 4)) != RC_OK) return rc;
-            RC_CUDA(c, cudaMemcpyAsync(c->st_idx.p, ev->session_idx, n_ev * 4, cudaMemcpyHostToDevice, c->stream));
+            if (!defer_inputs)
+                RC_CUDA(c, cudaMemcpyAsync(c->st_idx.p, ev->session_idx, n_ev * 4, cudaMemcpyHostToDevice,
+                                           c->stream));
             a.idx = static_cast<const uint32_t *>(c->st_idx.p);
+            r->host_idx = defer_inputs;
         }
     }
     r->user_dec = dec;
@@ -531,6 +548,99 @@ int build_nested(rc_ctx *c, const rc::StepArgs &a) {
     return RC_OK;
 }
 
+// ---- persistent chain with host-memory events, in pieces -----------------
+// The steps run as consecutive persistent launches over pieces of the event
+// sets (64 steps first, then four times the previous, up to 1,024): one copy
+// stream brings in every piece's events in order, another takes out each
+// piece's decisions, effects and state log once it is done, both while later
+// pieces run.  Each launch starts from the decision and the state the
+// previous one left, so the cohort sequence is the one of a single launch;
+// a link that would reach into the previous piece counts as absent and that
+// record is gathered from HBM, where the previous launch stored it.  Errors
+// report the step of the whole chain (dev->step_base).
+constexpr uint32_t kPieceFirst = 64, kPieceGrow = 4, kPieceMax = 1024, kPieceSlots = 1024;  // at most slots pieces
+
+bool pieces_apply(const Resolved &r, rc_mechanism mech) {
+    const rc::StepArgs &a = r.a;
+    return mech == RC_MECH_RESIDENT_PERSIST && a.K > 0 && a.n_steps >= 2u * kPieceFirst &&
+           a.n_sets == a.n_steps && (r.host_out || r.host_pay || r.host_idx);
+}
+
+int run_persist_pieces(rc_ctx *c, const Resolved &r) {
+    const rc::StepArgs &a0 = r.a;
+    const uint32_t n = a0.n_steps, K = a0.K;
+    const rc_events *ev = r.user_ev;
+    uint32_t cap = kPieceMax;  // at most kPieceSlots - 8 pieces
+    if ((n + cap - 1u) / cap > kPieceSlots - 8u) cap = (n + kPieceSlots - 9u) / (kPieceSlots - 8u);
+    std::vector<std::pair<uint32_t, uint32_t>> pieces;  // (first step, steps)
+    for (uint32_t first = 0, size = std::min(kPieceFirst, cap); first < n; first += pieces.back().second) {
+        pieces.emplace_back(first, std::min(size, n - first));
+        size = std::min(size * kPieceGrow, cap);
+    }
+    while (c->pipe_ev.size() < 2 * pieces.size() + 2) {
+        cudaEvent_t e;
+        RC_CUDA(c, cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
+        c->pipe_ev.push_back(e);
+    }
+    const cudaEvent_t start = c->pipe_ev[0], tail = c->pipe_ev[1];
+    // no copy of this call may overtake the work already queued on the context stream
+    RC_CUDA(c, cudaEventRecord(start, c->stream));
+    RC_CUDA(c, cudaStreamWaitEvent(c->copy_stream, start, 0));
+    RC_CUDA(c, cudaStreamWaitEvent(c->out_stream, start, 0));
+    for (size_t k = 0; k < pieces.size(); ++k) {
+        const size_t e0 = static_cast<size_t>(pieces[k].first) * K, ne = static_cast<size_t>(pieces[k].second) * K;
+        if (r.host_out)
+            RC_CUDA(c, cudaMemcpyAsync(const_cast<uint32_t *>(a0.outcome) + e0, ev->outcome + e0, ne * 4,
+                                       cudaMemcpyHostToDevice, c->copy_stream));
+        if (r.host_pay)
+            RC_CUDA(c, cudaMemcpyAsync(const_cast<uint8_t *>(a0.payload) + e0 * c->P, ev->payload + e0 * c->P,
+                                       ne * c->P, cudaMemcpyHostToDevice, c->copy_stream));
+        if (r.host_idx)
+            RC_CUDA(c, cudaMemcpyAsync(const_cast<uint32_t *>(a0.idx) + e0, ev->session_idx + e0, ne * 4,
+                                       cudaMemcpyHostToDevice, c->copy_stream));
+        RC_CUDA(c, cudaEventRecord(c->pipe_ev[2 + 2 * k], c->copy_stream));
+    }
+    uint32_t launches = 0;
+    for (size_t k = 0; k < pieces.size(); ++k) {
+        const uint32_t j0 = pieces[k].first, cnt = pieces[k].second;
+        const size_t e0 = static_cast<size_t>(j0) * K, ne = static_cast<size_t>(cnt) * K;
+        const cudaEvent_t in = c->pipe_ev[2 + 2 * k], done = c->pipe_ev[3 + 2 * k];
+        RC_CUDA(c, cudaStreamWaitEvent(c->stream, in, 0));
+        RC_CUDA(c, rc::launch_set_word(&c->dev->step_base, j0, c->stream));
+        rc::StepArgs a = a0;
+        a.outcome = a0.outcome + e0;
+        a.payload = a0.payload + e0 * c->P;
+        if (a0.idx) a.idx = a0.idx + e0;
+        a.n_sets = cnt;
+        a.n_steps = cnt;
+        a.trace = nullptr;
+        if (a0.decisions) a.decisions = a0.decisions + j0;
+        if (a0.effects) a.effects = a0.effects + e0 * 16;
+        if (a0.state_log) a.state_log = a0.state_log + e0 * c->SB;
+        int rc = run_persist(c, a);
+        if (rc != RC_OK) return rc;
+        launches += c->last_launches + 1u;  // the piece's chain, and its step base
+        RC_CUDA(c, cudaEventRecord(done, c->stream));
+        RC_CUDA(c, cudaStreamWaitEvent(c->out_stream, done, 0));
+        if (r.host_dec)
+            RC_CUDA(c, cudaMemcpyAsync(r.user_dec + j0, a.decisions, static_cast<size_t>(cnt) * 4,
+                                       cudaMemcpyDeviceToHost, c->out_stream));
+        if (r.host_eff)
+            RC_CUDA(c, cudaMemcpyAsync(static_cast<uint8_t *>(r.user_eff) + e0 * 16, a.effects, ne * 16,
+                                       cudaMemcpyDeviceToHost, c->out_stream));
+        if (r.host_log)
+            RC_CUDA(c, cudaMemcpyAsync(static_cast<uint8_t *>(r.user_log) + e0 * c->SB, a.state_log, ne * c->SB,
+                                       cudaMemcpyDeviceToHost, c->out_stream));
+    }
+    // the context stream ends after the last copies (the input stream is
+    // done once the last piece started); the step base returns to 0
+    RC_CUDA(c, cudaEventRecord(tail, c->out_stream));
+    RC_CUDA(c, cudaStreamWaitEvent(c->stream, tail, 0));
+    RC_CUDA(c, rc::launch_set_word(&c->dev->step_base, 0u, c->stream));
+    c->last_launches = launches + 1u;
+    return RC_OK;
+}
+
 int run_nested(rc_ctx *c, const rc::StepArgs &a) {
     if (!(c->nested.valid && c->nested.key == key_of(a, 3, 0))) {
         int rc = build_nested(c, a);
@@ -620,6 +730,8 @@ int rc_init(rc_ctx **out, uint32_t S, const uint8_t *table, uint32_t state_bytes
         c->no_prod = q && q[0] == '1';
         const char *pr = std::getenv("RC_PAIR");
         c->use_pair = pr && pr[0] == '1';
+        const char *np = std::getenv("RC_NO_PIECES");
+        c->no_pieces = np && np[0] == '1';
         const char *gl = std::getenv("RC_NO_GRID_LINK");
         c->no_grid_link = gl && gl[0] == '1';
         const char *cl = std::getenv("RC_NO_CLUSTER");
@@ -654,6 +766,9 @@ int rc_init(rc_ctx **out, uint32_t S, const uint8_t *table, uint32_t state_bytes
         return bail(e);
     if ((e = cudaEventCreate(&c->ev_start)) != cudaSuccess) return bail(e);
     if ((e = cudaEventCreate(&c->ev_stop)) != cudaSuccess) return bail(e);
+    if ((e = cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking)) != cudaSuccess) return bail(e);
+    if ((e = cudaStreamCreateWithFlags(&c->out_stream, cudaStreamNonBlocking)) != cudaSuccess) return bail(e);
+
     std::memset(c->h_pinned, 0, 64);
     *out = c;
     return RC_OK;
@@ -690,8 +805,23 @@ int rc_chain(rc_ctx *c, uint32_t n_steps, rc_mechanism mech, void *state, const 
     if (floor && (!decisions || !is_host_ptr(decisions)))
         return fail(c, RC_E_INVAL, "the floor replays a route sequence given in host memory (decisions_out)");
     Resolved r;
-    int rc = resolve(c, state, ev, K, n_steps, decisions, effects, state_log, floor, &r);
+    const bool may_piece = mech == RC_MECH_RESIDENT_PERSIST && ev && ev->n_sets == n_steps && !c->no_pieces;
+    int rc = resolve(c, state, ev, K, n_steps, decisions, effects, state_log, floor, &r, may_piece);
     if (rc != RC_OK) return rc;
+    const bool pieces = may_piece && pieces_apply(r, mech);
+    if (may_piece && !pieces) {
+        // inputs staged whole after all
+        const size_t n_ev = static_cast<size_t>(r.a.n_sets) * K;
+        if (r.host_out)
+            RC_CUDA(c, cudaMemcpyAsync(const_cast<uint32_t *>(r.a.outcome), ev->outcome, n_ev * 4,
+                                       cudaMemcpyHostToDevice, c->stream));
+        if (r.host_pay)
+            RC_CUDA(c, cudaMemcpyAsync(const_cast<uint8_t *>(r.a.payload), ev->payload, n_ev * c->P,
+                                       cudaMemcpyHostToDevice, c->stream));
+        if (r.host_idx)
+            RC_CUDA(c, cudaMemcpyAsync(const_cast<uint32_t *>(r.a.idx), ev->session_idx, n_ev * 4,
+                                       cudaMemcpyHostToDevice, c->stream));
+    }
     if (floor) r.a.decisions = nullptr;
     c->last_ms = 0.0;
     c->last_launches = 0;
@@ -710,7 +840,7 @@ int rc_chain(rc_ctx *c, uint32_t n_steps, rc_mechanism mech, void *state, const 
         switch (mech) {
             case RC_MECH_HOST_RT: rc = run_host_rt(c, r.a); break;
             case RC_MECH_RESIDENT_COND: rc = run_cond(c, r.a); break;
-            case RC_MECH_RESIDENT_PERSIST: rc = run_persist(c, r.a); break;
+            case RC_MECH_RESIDENT_PERSIST: rc = pieces ? run_persist_pieces(c, r) : run_persist(c, r.a); break;
             case RC_MECH_FIXED_NESTED: rc = run_nested(c, r.a); break;
             case RC_MECH_FLOOR: rc = run_floor(c, r.a, decisions); break;
             default: rc = fail(c, RC_E_INVAL, "unknown mechanism");
@@ -718,8 +848,10 @@ int rc_chain(rc_ctx *c, uint32_t n_steps, rc_mechanism mech, void *state, const 
         if (rc != RC_OK) return rc;
     }
     RC_CUDA(c, cudaEventRecord(c->ev_stop, c->stream));
-    rc = copy_back(c, r, n_steps);
-    if (rc != RC_OK) return rc;
+    if (!pieces) {
+        rc = copy_back(c, r, n_steps);
+        if (rc != RC_OK) return rc;
+    }
     rc = finish(c);
     float ms = 0.f;
     if (cudaEventElapsedTime(&ms, c->ev_start, c->ev_stop) == cudaSuccess) c->last_ms = ms;
@@ -739,6 +871,13 @@ int rc_free(rc_ctx *c) {
     if (c->h_pinned) cudaFreeHost(c->h_pinned);
     if (c->ev_start) cudaEventDestroy(c->ev_start);
     if (c->ev_stop) cudaEventDestroy(c->ev_stop);
+    for (cudaStream_t st : {c->copy_stream, c->out_stream}) {
+        if (st) {
+            cudaStreamSynchronize(st);
+            cudaStreamDestroy(st);
+        }
+    }
+    for (cudaEvent_t e : c->pipe_ev) cudaEventDestroy(e);
     delete c;
     return RC_OK;
 }

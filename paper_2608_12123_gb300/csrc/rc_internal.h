@@ -20,7 +20,8 @@ struct alignas(256) DevBlock {
     uint32_t count;         // odd-key count of a multi-CTA step
     uint32_t skip_arrival;  // test hook: CTA 1 skips its first grid-barrier arrival
     uint32_t abort;         // set by a CTA whose bounded wait ran out
-    uint32_t pad0[3];
+    uint32_t step_base;     // added to the step of a latched error (chains run in pieces)
+    uint32_t pad0[2];
     uint64_t wait_ns;       // device spin-wait limit (ns of %globaltimer)
     unsigned long long slot[3];  // grid-barrier words of the persistent grid kernel
     uint32_t countdown;     // launch-floor probe: WHILE iterations left
@@ -185,6 +186,8 @@ cudaError_t launch_chain_owned(const StepArgs &a, int state_bytes, int payload_b
 cudaError_t launch_seg_step(const SegArgs &a, int state_bytes, int payload_bytes, cudaStream_t s);
 
 // Writes decisions[0..n) = 0 and sel = 0 (an empty cohort decides 0).
+// Writes one word in stream order (a one-thread kernel).
+cudaError_t launch_set_word(uint32_t *p, uint32_t v, cudaStream_t s);
 cudaError_t launch_empty_cohorts(const StepArgs &a, cudaStream_t s);
 
 // Fixed-nested control: a one-thread kernel that device-launches `child`.

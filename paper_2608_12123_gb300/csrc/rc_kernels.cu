@@ -117,7 +117,7 @@ __device__ __forceinline__ void mix_acc(uint4 (&r)[SB / 16], uint64_t rk) {
 
 __device__ __forceinline__ void latch_error(DevBlock *dev, uint32_t code, uint32_t step, uint32_t member) {
     if (atomicCAS(&dev->err, 0u, code) == 0u) {
-        dev->err_step = step;
+        dev->err_step = step + dev->step_base;
         dev->err_member = member;
     }
 }
@@ -3097,6 +3097,9 @@ __global__ void k_launch_child(cudaGraphExec_t child, DevBlock *dev) {
     }
 }
 
+// One word written in stream order (the step base of a chain run in pieces).
+__global__ void k_set_word(uint32_t *p, uint32_t v) { *p = v; }
+
 __global__ void k_empty() {}
 
 __global__ void k_countdown(DevBlock *dev, cudaGraphConditionalHandle h) {
@@ -3828,6 +3831,11 @@ cudaError_t launch_empty_cohorts(const StepArgs &a, cudaStream_t s) {
     StepArgs aa = a;
     void *args[] = {&aa};
     return cudaLaunchKernel(reinterpret_cast<const void *>(&k_empty_cohorts), dim3(1), dim3(256), args, 0, s);
+}
+
+cudaError_t launch_set_word(uint32_t *p, uint32_t v, cudaStream_t s) {
+    k_set_word<<<1, 1, 0, s>>>(p, v);
+    return cudaGetLastError();
 }
 
 const void *launcher_kernel() { return reinterpret_cast<const void *>(&k_launch_child); }

@@ -89,6 +89,57 @@ def test_host_buffers_give_identical_results(g, rc):
         g.assert_same(got, want, f"host buffers {name}")
 
 
+@pytest.mark.parametrize("K,N,n,SB,P,identity", [(256, 300, 128, 16, 64, False), (256, 259, 1000, 16, 64, False),
+                                                   (64, 70, 400, 64, 128, False), (40, 40, 330, 16, 32, True),
+                                                   (2048, 2100, 130, 16, 64, False), (8192, 1 << 20, 129, 64, 128, False)])
+def test_host_buffers_in_pieces(g, rc, K, N, n, SB, P, identity):
+    """A persistent chain over host-memory events, one cohort per step, runs in
+    pieces (64 steps, then four times the previous up to 1,024) with the
+    copies of later pieces overlapping the current one; sessions recur across the piece
+    boundaries (N close to K).  Every output equals the oracle's, and the
+    whole chain counts two launches per piece where a link pass precedes the
+    chain."""
+    import torch
+    S = 256 if SB == 64 else 64
+    tables, state0, outc, pay, idx = _inputs(110 + K % 11 + n, K, S, SB, P, n, N=N)
+    if identity:
+        idx = None
+    want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=1)
+    got = g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K, sel0=1, host_buffers=True)
+    g.assert_same(got, want, f"pieces K={K} N={N} n={n}")
+    pieces, first, size = 0, 0, 64
+    while first < n:
+        first += min(size, n - first)
+        size = min(4 * size, 1024)
+        pieces += 1
+    ctx = rc.rc_init(S, tables, SB, P, K, N, torch.cuda.current_stream())
+    try:
+        state = g.dev(state0.copy())
+        ev = rc.make_events(np.ascontiguousarray(outc), np.ascontiguousarray(pay),
+                            None if idx is None else np.ascontiguousarray(idx), payload_bytes=P, n_sets=n)
+        dec = np.zeros(n, np.uint32)
+        rc.rc_chain(ctx, n, rc.RC_MECH_RESIDENT_PERSIST, state, ev, K, dec)
+        _, launches = rc.rc_last_chain_stats(ctx)
+        # per piece: its step base, then the chain (with its pre-pass); one
+        # more write returns the step base to 0
+        per_piece = (launches - 1) // pieces
+        assert launches == per_piece * pieces + 1 and per_piece in (2, 3, 4), (launches, pieces)
+    finally:
+        rc.rc_free(ctx)
+
+
+def test_error_step_counts_from_the_chain_start_in_pieces(g, rc):
+    """A latched error in a later piece reports its step in the whole chain."""
+    K, S, SB, P, n = 64, 16, 16, 32, 200
+    tables, state0, outc, pay, idx = _inputs(131, K, S, SB, P, n, N=500)
+    o2 = outc.copy()
+    o2[150, 7] = 8  # step 150 lies in the second piece (64 + 256 + ...)
+    with pytest.raises(rc.RcError) as e:
+        g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, o2, pay, idx, n, K, host_buffers=True)
+    assert e.value.code == rc.RC_E_STATE
+    assert "step 150, member 7" in str(e.value), str(e.value)
+
+
 def test_cohort_step_api_carries_the_flag_and_checks_deadlines(g, rc):
     import torch
     K, S, SB, P, n = 100, 32, 16, 32, 25
