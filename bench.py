@@ -347,7 +347,7 @@ def native(args):
 
         alg_bytes = H * K * BYTES_PER_TRANSITION_C2
         ach = alg_bytes / (step_ms * 1e-3) / 1e9
-        traffic = ncu_traffic("k_chain_cta_prod<16,64>", H * K)
+        traffic = ncu_traffic("k_chain_cta_pair<16,64>", H * K)
         out.update({
             "metric": METRIC, "value": round(value, 4), "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(step_ms, 4), "higher_is_better": False,
@@ -375,7 +375,8 @@ def native(args):
                                 "vs_launch_sync": round(us_inv / floor_probe["launch_sync"], 3)},
             "roofline": {"bound": "hbm", "achieved": round(ach, 3), "peak": hbm_peak, "unit": "GB/s",
                          "frac": round(ach / hbm_peak, 5), "traffic": traffic,
-                         "kernel": "k_chain_cta_prod<16,64> (one launch = 1,000 steps x 256 members, after the k_link pass)",
+                         "kernel": "k_chain_cta_pair<16,64> (one launch = 1,000 steps x 256 members, two per block "
+                                   "barrier, after the k_link_reach pass)",
                          "peak_source": f"{peak_src} hbm_gbs",
                          "note": "K=256 steps are latency-bound: see latency_x_floor"},
             "e2e": {"value": round(e2e_us, 4), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},

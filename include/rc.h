@@ -39,8 +39,14 @@
  *   - "Device pointer" means memory the GPU of the context can address
  *     (cudaMalloc / torch CUDA tensors).  Event and output buffers may also be
  *     host memory (pageable or pinned): the library then copies them through
- *     its own device staging buffers on the context stream, inside the call.
- *     The state array must be device memory.
+ *     its own device staging buffers, inside the call.  A persistent chain
+ *     with one cohort per step (n_sets == n_steps, at least 128 steps) over
+ *     host-memory events runs as consecutive persistent launches over pieces
+ *     of the steps (64, then four times the previous, up to 1,024), with
+ *     the copies of later pieces' events and of earlier pieces' outputs on
+ *     two library streams overlapping the running piece; the results are the
+ *     ones of one launch (set RC_NO_PIECES=1 in the environment to stage
+ *     whole).  The state array must be device memory.
  *   - All buffers passed in stay owned by the caller; the library owns the
  *     context, its device copy of the tables, the decision flag, counters,
  *     staging buffers, pinned host words and CUDA graphs.

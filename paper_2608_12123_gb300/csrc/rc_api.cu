@@ -95,7 +95,7 @@ struct rc_ctx {
     bool no_pipe = false;   // RC_NO_PIPE=1 selects the plain single-CTA kernel
     bool no_link = false;   // RC_NO_LINK=1 turns off the linked single-CTA kernels
     bool no_prod = false;   // RC_NO_PROD=1 keeps the linked kernel without a producer warp
-    bool use_pair = false;  // RC_PAIR=1 selects the single-CTA chain keying two steps per barrier
+    bool no_pair = false;   // RC_NO_PAIR=1 turns off the single-CTA chain keying two steps per barrier
     bool no_pieces = false; // RC_NO_PIECES=1 stages host-memory events whole (no pieces)
     bool no_grid_link = false;  // RC_NO_GRID_LINK=1 turns off the grid chain split by links
     bool no_cluster = false;    // RC_NO_CLUSTER=1 turns off the cluster chain (512 < K <= 8192)
@@ -442,7 +442,7 @@ int run_persist(rc_ctx *c, const rc::StepArgs &a) {
             return RC_OK;
         }
     }
-    if (a.idx && c->use_pair && !c->no_pipe && !c->no_link) {
+    if (a.idx && !c->no_pair && !c->no_pipe && !c->no_link && !c->no_prod) {
         size_t smem = 0;
         alignas(8) unsigned char shape[16];
         if (rc::chain_cta_pair_plan(c->SB, c->P, a.K, c->S, c->n_sessions, c->tab_stride, &smem, shape)) {
@@ -470,7 +470,7 @@ int run_persist(rc_ctx *c, const rc::StepArgs &a) {
     }
     if (a.K <= 1024u) {
         bool launched = false;
-        if (!c->no_pipe) RC_CUDA(c, rc::launch_chain_cta_fast(a, c->SB, c->P, c->stream, &launched));
+        if (!c->no_pipe) RC_CUDA(c, rc::launch_chain_cta_fast(a, c->SB, c->P, c->stream, &launched, !c->no_pair));
         if (launched) return RC_OK;
         if (a.K <= 512u) {
             RC_CUDA(c, rc::launch_chain_cta(a, c->SB, c->P, c->stream));
@@ -728,8 +728,8 @@ int rc_init(rc_ctx **out, uint32_t S, const uint8_t *table, uint32_t state_bytes
         c->no_link = z && z[0] == '1';
         const char *q = std::getenv("RC_NO_PROD");
         c->no_prod = q && q[0] == '1';
-        const char *pr = std::getenv("RC_PAIR");
-        c->use_pair = pr && pr[0] == '1';
+        const char *pr = std::getenv("RC_NO_PAIR");
+        c->no_pair = pr && pr[0] == '1';
         const char *np = std::getenv("RC_NO_PIECES");
         c->no_pieces = np && np[0] == '1';
         const char *gl = std::getenv("RC_NO_GRID_LINK");

@@ -106,10 +106,11 @@ cudaError_t launch_step(const StepArgs &a, int state_bytes, int payload_bytes, i
 // Persistent chains.  The single-CTA form takes K <= 512; the grid form is a
 // cooperative launch of `grid` CTAs.
 cudaError_t launch_chain_cta(const StepArgs &a, int state_bytes, int payload_bytes, cudaStream_t s);
-// Pipelined single-CTA chain for identity sessions (records in registers).
-// *launched is false when it does not apply.
+// Pipelined single-CTA chain for identity sessions (records in registers);
+// with two_steps and K <= 512, two steps per block barrier.  *launched is
+// false when it does not apply.
 cudaError_t launch_chain_cta_fast(const StepArgs &a, int state_bytes, int payload_bytes, cudaStream_t s,
-                                  bool *launched);
+                                  bool *launched, bool two_steps);
 // Single-CTA chains with explicit indices and the record gather ahead of its
 // step (K <= 512): launch_link fills lnk (n_sets * K words) with each
 // member's position in the two previous cohorts, then the chain runs (the

@@ -555,6 +555,162 @@ __global__ void __launch_bounds__(1024, 1) k_chain_cta_ident(StepArgs a) {
 }
 
 // ---------------------------------------------------------------------------
+// Persistent chain, one CTA, member m = session m (K <= 512), two steps per
+// block barrier.  Thread m holds its session's record in registers for the
+// whole chain.  The key of step j reads the state the session left in step
+// j - 1, T_sel(j-1)[x][o] with sel(j-1) = d(j-2); so once d(2r-1) is known the
+// keys of steps 2r and 2r+1 are two independent hash chains of one thread,
+// and one block barrier counts both (the two counts packed in one word per
+// warp).  The record update of step 2r+1 needs d(2r) and is applied at the
+// start of the next region.  Outcomes and payload rows come through a ring of
+// per-thread asynchronous copies D steps deep (two steps consumed per region,
+// D + 2 slots).
+// ---------------------------------------------------------------------------
+template <int SB, int P, int D>
+__global__ void __launch_bounds__(512, 1) k_chain_cta_ident2(StepArgs a) {
+    static_assert(D >= 2, "two steps per region");
+    constexpr uint32_t RD = D + 2;
+    constexpr uint32_t NC = P / 16;
+    constexpr int NV = SB / 16;
+    extern __shared__ __align__(16) uint8_t dsm[];
+    __shared__ uint32_t warp_odd[2][16];
+    const uint32_t K = a.K;
+    const uint32_t Kp = (K + 3u) & ~3u;
+    const uint32_t tid = threadIdx.x;
+    const uint32_t nw = (blockDim.x + 31u) / 32u;
+    uint8_t *tab = dsm;
+    uint32_t *out_r = reinterpret_cast<uint32_t *>(dsm + 2 * a.tab_stride);
+    uint4 *pay_r = reinterpret_cast<uint4 *>(out_r + RD * Kp);
+    stage_tables(tab, a.tables, a.tab_stride, 2, 0);
+    const bool act = tid < K;
+    const uint32_t m = tid;
+    const uint32_t nst = a.n_steps;
+    const bool in_range = m < a.n_sessions;
+    uint4 r[NV];
+#pragma unroll
+    for (int k = 0; k < NV; ++k) r[k] = make_uint4(0, 0, 0, 0);
+    if (act && in_range) {
+        const uint4 *rp = reinterpret_cast<const uint4 *>(a.state + static_cast<size_t>(m) * SB);
+#pragma unroll
+        for (int k = 0; k < NV; ++k) r[k] = rp[k];
+    }
+    auto issue_data = [&](uint32_t j) {
+        if (act && j < nst) {
+            const size_t e = static_cast<size_t>(j % a.n_sets) * K + m;
+            cp_async4(&out_r[(j % RD) * Kp + m], a.outcome + e);
+            const uint4 *src = reinterpret_cast<const uint4 *>(a.payload + e * P);
+            uint4 *ring = pay_r + (j % RD) * Kp * NC;
+#pragma unroll
+            for (uint32_t k = 0; k < NC; ++k) cp_async16(ring + pay_chunk<P>(m, k), src + k);
+        }
+        cp_async_commit();
+    };
+    // this thread's record update for step n under decision sel (a valid member)
+    auto apply = [&](uint32_t n, uint32_t sel, uint32_t o, uint64_t rk) {
+        const uint32_t x = r[0].x;
+        const uint32_t y = tab[sel * a.tab_stride + x * 8u + o];
+        r[0].x = y;
+        r[0].y = r[0].y + 1u;
+        mix_acc<SB>(r, rk);
+        const size_t slot = static_cast<size_t>(n) * K + m;
+        if (a.effects) {
+            uint4 e;
+            e.x = static_cast<uint32_t>(rk);
+            e.y = static_cast<uint32_t>(rk >> 32);
+            e.z = m;
+            e.w = y | (o << 16) | (sel << 24);
+            __stcs(reinterpret_cast<uint4 *>(a.effects) + slot, e);
+        }
+        if (a.state_log) {
+            uint4 *lp = reinterpret_cast<uint4 *>(a.state_log + slot * SB);
+#pragma unroll
+            for (int k = 0; k < NV; ++k) __stcs(lp + k, r[k]);
+        }
+    };
+    for (uint32_t j = 0; j < D; ++j) issue_data(j);
+    __syncthreads();
+    uint32_t sel_a = ld_volatile_u32(&a.dev->sel) & 1u;  // decision for step 2r: d(2r-1)
+    uint32_t sel_b = 0;                                  // decision for step 2r-1: d(2r-2)
+    bool pend = false;                                   // step 2r-1 keyed, record update pending
+    uint32_t pend_o = 0;
+    uint64_t pend_rk = 0;
+    uint32_t last = sel_a;  // the decision of the last step decided
+    for (uint32_t ja = 0; ja < nst; ja += 2u) {
+        const uint32_t jb = ja + 1u;
+        const bool has_b = jb < nst;
+        cp_async_wait<D - 2>();  // this thread's data of steps ja and jb
+        if (pend) apply(ja - 1u, sel_b, pend_o, pend_rk);
+        pend = false;
+        uint32_t odd_a = 0, odd_b = 0;
+        if (act) {
+            const uint32_t o_a = out_r[(ja % RD) * Kp + m];
+            const uint32_t o_b = has_b ? out_r[(jb % RD) * Kp + m] : 0u;
+            if (!in_range) {
+                latch_error(a.dev, DEV_E_INDEX, ja, m);
+                if (has_b) latch_error(a.dev, DEV_E_INDEX, jb, m);
+            } else {
+                const uint32_t x_a = r[0].x;
+                const bool ok_a = x_a < a.S && o_a < 8u;
+                if (!ok_a) latch_error(a.dev, DEV_E_STATE, ja, m);
+                const uint32_t x_b = ok_a ? static_cast<uint32_t>(tab[sel_a * a.tab_stride + x_a * 8u + o_a]) : x_a;
+                const bool ok_b = has_b && x_b < a.S && o_b < 8u;
+                if (has_b && !ok_b) latch_error(a.dev, DEV_E_STATE, jb, m);
+                uint4 pa[NC], pb[NC];
+                const uint4 *ra = pay_r + (ja % RD) * Kp * NC;
+                const uint4 *rb = pay_r + (jb % RD) * Kp * NC;
+#pragma unroll
+                for (uint32_t k = 0; k < NC; ++k) {
+                    pa[k] = ra[pay_chunk<P>(m, k)];
+                    pb[k] = ok_b ? rb[pay_chunk<P>(m, k)] : make_uint4(0, 0, 0, 0);
+                }
+                // two independent key chains (the second on a valid dummy when unused)
+                const uint64_t rk_a = route_key<P>(ok_a ? x_a : 0u, ok_a ? o_a : 0u, pa);
+                const uint64_t rk_b = route_key<P>(ok_b ? x_b : 0u, ok_b ? o_b : 0u, pb);
+                if (ok_a) {
+                    apply(ja, sel_a, o_a, rk_a);
+                    odd_a = static_cast<uint32_t>(rk_a & 1u);
+                }
+                if (ok_b) {
+                    pend = true;
+                    pend_o = o_b;
+                    pend_rk = rk_b;
+                    odd_b = static_cast<uint32_t>(rk_b & 1u);
+                }
+            }
+        }
+        issue_data(ja + D);
+        issue_data(ja + D + 1u);
+        const uint32_t ca = __popc(__ballot_sync(0xffffffffu, odd_a != 0u));
+        const uint32_t cb = __popc(__ballot_sync(0xffffffffu, odd_b != 0u));
+        const uint32_t rr = (ja >> 1) & 1u;
+        if ((tid & 31u) == 0) warp_odd[rr][tid >> 5] = ca | (cb << 16);
+        __syncthreads();
+        uint32_t total = 0;
+        for (uint32_t w = 0; w < nw; ++w) total += warp_odd[rr][w];
+        const uint32_t da = (total & 0xFFFFu) > K / 2u ? 1u : 0u;
+        const uint32_t db = (total >> 16) > K / 2u ? 1u : 0u;
+        if (tid == 0 && a.decisions) {
+            a.decisions[ja] = da;
+            if (has_b) a.decisions[jb] = db;
+        }
+        sel_b = da;
+        sel_a = db;
+        last = has_b ? db : da;
+    }
+    if (pend) apply(nst - 1u, sel_b, pend_o, pend_rk);
+    cp_async_wait<0>();
+    if (act && in_range) {
+        uint4 *rp = reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(m) * SB);
+#pragma unroll
+        for (int k = 0; k < NV; ++k) rp[k] = r[k];
+    }
+    if (tid == 0) {
+        if (nst > 0) a.dev->sel = last;
+        a.dev->step = nst;
+    }
+}
+
+// ---------------------------------------------------------------------------
 // Persistent chain, cooperative grid (any K): each CTA owns a grid-stride
 // slice of members.  Per step, after a block barrier, thread 0 of each CTA
 // adds (1 << 32 | odd count) to the step's barrier word with release
@@ -3170,6 +3326,17 @@ size_t ident_smem(uint32_t K, int P, int D, uint32_t tab_stride) {
     const size_t Kp = (K + 3u) & ~3u, RD = D + 1;
     return 2 * tab_stride + RD * Kp * 4 + RD * Kp * P;
 }
+const void *ident2_fn_rt(int SB, int P, int D) {
+    return dispatch(SB, P, [&](auto b, auto q) {
+        constexpr int B = decltype(b)::value, Q = decltype(q)::value;
+        return D == 4 ? reinterpret_cast<const void *>(&k_chain_cta_ident2<B, Q, 4>)
+                      : reinterpret_cast<const void *>(&k_chain_cta_ident2<B, Q, 2>);
+    });
+}
+size_t ident2_smem(uint32_t K, int P, int D, uint32_t tab_stride) {
+    const size_t Kp = (K + 3u) & ~3u, RD = D + 2;
+    return 2 * tab_stride + RD * Kp * 4 + RD * Kp * P;
+}
 int max_optin_smem() {
     int dev = 0, v = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 0;
@@ -3178,13 +3345,26 @@ int max_optin_smem() {
 }
 }  // namespace
 
-cudaError_t launch_chain_cta_fast(const StepArgs &a, int SB, int P, cudaStream_t s, bool *launched) {
+cudaError_t launch_chain_cta_fast(const StepArgs &a, int SB, int P, cudaStream_t s, bool *launched,
+                                  bool two_steps) {
     *launched = false;
     const uint32_t K = a.K;
     if (K == 0 || K > 1024u) return cudaSuccess;
     const size_t cap = static_cast<size_t>(max_optin_smem());
     const uint32_t threads = ((K + 31u) / 32u) * 32u;
     StepArgs aa = a;
+    if (!a.idx && two_steps && K <= 512u) {
+        for (int D : {4, 2}) {
+            const size_t smem = ident2_smem(K, P, D, a.tab_stride);
+            if (smem > cap) continue;
+            const void *fn = ident2_fn_rt(SB, P, D);
+            cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+            if (e != cudaSuccess) return e;
+            void *args[] = {&aa};
+            *launched = true;
+            return cudaLaunchKernel(fn, dim3(1), dim3(threads), args, smem, s);
+        }
+    }
     if (!a.idx) {
         for (int D : {4, 2, 1}) {
             const size_t smem = ident_smem(K, P, D, a.tab_stride);

@@ -285,12 +285,13 @@ def test_grid_barrier_wait_is_bounded_every_grid_kernel(g, rc, monkeypatch, kern
 def test_small_cohort_repeated_sessions(g, rc, monkeypatch, kernel, P, K, N):
     """Sessions that recur in consecutive steps at other member positions: each
     persistent kernel must see the records the previous step wrote ("pair":
-    the single-CTA chain keying two steps per barrier, K <= 256 and P <= 64)."""
+    the single-CTA chain keying two steps per barrier, taken where it applies,
+    K <= 256 and P <= 64; "prod" with it turned off)."""
     monkeypatch.setenv("RC_OWNED", "1" if kernel == "owned" else "0")
     monkeypatch.setenv("RC_SPLIT", "1" if kernel == "split" else "0")
     monkeypatch.setenv("RC_NO_PIPE", "1" if kernel == "plain" else "0")
     monkeypatch.setenv("RC_NO_PROD", "1" if kernel == "link" else "0")
-    monkeypatch.setenv("RC_PAIR", "1" if kernel == "pair" else "0")
+    monkeypatch.setenv("RC_NO_PAIR", "0" if kernel == "pair" else "1")
     tables, state0, outc, pay, idx = _inputs(60 + K % 13 + P, K, 64, 16, P, 40, N=N)
     n = 40
     want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=1)
@@ -298,16 +299,22 @@ def test_small_cohort_repeated_sessions(g, rc, monkeypatch, kernel, P, K, N):
     g.assert_same(got, want, f"{kernel} K={K} N={N} P={P}")
 
 
-@pytest.mark.parametrize("pipe", [True, False])
-@pytest.mark.parametrize("SB,P,K", [(16, 32, 32), (16, 32, 256), (64, 128, 256), (64, 64, 700), (16, 128, 1024)])
-def test_single_cta_identity_sessions(g, rc, monkeypatch, pipe, SB, P, K):
-    monkeypatch.setenv("RC_NO_PIPE", "0" if pipe else "1")
+@pytest.mark.parametrize("n", [30, 31])
+@pytest.mark.parametrize("mode", ["two", "one", "plain"])
+@pytest.mark.parametrize("SB,P,K", [(16, 32, 32), (16, 32, 256), (64, 128, 256), (64, 64, 700), (16, 128, 1024),
+                                    (16, 64, 500), (64, 32, 8)])
+def test_single_cta_identity_sessions(g, rc, monkeypatch, mode, SB, P, K, n):
+    """Member m = session m: the record stays in registers.  "two": two steps
+    per block barrier (K <= 512), "one": one step per barrier, "plain": the
+    plain single-CTA kernel.  An odd step count leaves a last region of one
+    step."""
+    monkeypatch.setenv("RC_NO_PIPE", "1" if mode == "plain" else "0")
+    monkeypatch.setenv("RC_NO_PAIR", "1" if mode == "one" else "0")
     S = 256 if SB == 64 else 128
-    tables, state0, outc, pay, idx = _inputs(80 + K % 17, K, S, SB, P, 30)
-    n = 30
-    want = g.run_oracle(tables, state0, outc, pay, idx, n)
-    got = g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K)
-    g.assert_same(got, want, f"identity pipe={pipe} SB={SB} P={P} K={K}")
+    tables, state0, outc, pay, idx = _inputs(80 + K % 17, K, S, SB, P, n)
+    want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=n % 2)
+    got = g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K, sel0=n % 2)
+    g.assert_same(got, want, f"identity {mode} SB={SB} P={P} K={K} n={n}")
 
 
 @pytest.mark.parametrize("kernel", ["pair", "prod"])
@@ -330,7 +337,7 @@ def test_linked_single_cta_ring_wraps(g, rc, monkeypatch, SB, P, K, extra, want_
     records and 128-byte payloads do not fit its rings and take the plain
     single-CTA kernel (one launch)."""
     import torch
-    monkeypatch.setenv("RC_PAIR", "1" if kernel == "pair" else "0")
+    monkeypatch.setenv("RC_NO_PAIR", "0" if kernel == "pair" else "1")
     S = 256 if SB == 64 else 64
     N = K + extra
     tables, state0, outc, pay, idx = _inputs(90 + n_sets + K % 7, K, S, SB, P, n_sets, N=N)
