@@ -225,6 +225,23 @@ def test_launch_floor_probes_run(g, rc):
         rc.rc_free(ctx)
 
 
+@pytest.mark.parametrize("n_sets", [1, 2, 3, 4, 7])
+@pytest.mark.parametrize("SB,P,K,N", [(64, 128, 2056, 2100), (16, 64, 4104, 12000), (64, 32, 1032, 1032)])
+def test_grid_link_records_stored_early_and_late(g, rc, monkeypatch, n_sets, SB, P, K, N):
+    """The grid chain split by links over many steps: sessions recurring at
+    distances 1, 2, 3 and more (rings of 1 to 7 cohorts drawn from N near K)
+    must see every earlier record, whether it reaches them through the
+    linked gather after the barrier or the unlinked gather run ahead while the
+    barrier is awaited."""
+    monkeypatch.setenv("RC_NO_CLUSTER", "1")
+    S = 256 if SB == 64 else 64
+    tables, state0, outc, pay, idx = _inputs(140 + n_sets + K % 7, K, S, SB, P, n_sets, N=N)
+    n = 14
+    want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=1)
+    got = g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K, sel0=1)
+    g.assert_same(got, want, f"grid link n_sets={n_sets} SB={SB} P={P} K={K} N={N}")
+
+
 @pytest.mark.parametrize("kernel", ["link", "owned", "split", "tma", "plain"])
 @pytest.mark.parametrize("SB,P", [(16, 32), (16, 64), (64, 128), (64, 32)])
 @pytest.mark.parametrize("K,N,identity", [(1032, 5000, False), (4104, 9001, False), (4104, 4200, False),
