@@ -399,6 +399,8 @@ int run_cond(rc_ctx *c, const rc::StepArgs &a) {
 }
 
 // ---- device resident: persistent kernel ------------------------------------
+constexpr uint32_t kPairMinSteps = 64;
+
 int run_persist(rc_ctx *c, const rc::StepArgs &a) {
     if (a.idx && c->use_owned && c->coop && static_cast<uint64_t>(a.n_sets) * a.K < (1ull << 31) - 1024u) {
         int grid = 0;
@@ -442,7 +444,9 @@ int run_persist(rc_ctx *c, const rc::StepArgs &a) {
             return RC_OK;
         }
     }
-    if (a.idx && !c->no_pair && !c->no_pipe && !c->no_link && !c->no_prod) {
+    // the two-step chain pays a heavier start (eight-cohort link pass, larger
+    // prologue: about 5 to 7 us); it is taken for chains of kPairMinSteps or more
+    if (a.idx && !c->no_pair && !c->no_pipe && !c->no_link && !c->no_prod && a.n_steps >= kPairMinSteps) {
         size_t smem = 0;
         alignas(8) unsigned char shape[16];
         if (rc::chain_cta_pair_plan(c->SB, c->P, a.K, c->S, c->n_sessions, c->tab_stride, &smem, shape)) {

@@ -1576,8 +1576,10 @@ __global__ void __launch_bounds__(544, 1)
 // nearest earlier cohort holding the same session (cohorts taken cyclically,
 // as a chain walks them) and its position q there, packed as t << 16 | q; 0
 // when none of the D cohorts before holds the session or the index is out of
-// range.  One CTA per cohort, one open-addressing table of SLOTS slots per
-// earlier cohort (at most SLOTS / 2 keys: K <= SLOTS / 2).
+// range.  One CTA per cohort and one open-addressing table of SLOTS slots
+// (at most SLOTS / 2 keys: D * K <= SLOTS / 2): every member of the D earlier
+// cohorts is inserted under its session, the packed value kept by atomicMin
+// (the nearest cohort wins), and each member of cohort j probes once.
 // ---------------------------------------------------------------------------
 constexpr uint32_t kPairD = 8;  // reach of k_chain_cta_pair's links
 
@@ -1586,24 +1588,40 @@ __global__ void __launch_bounds__(512) k_link_reach(const uint32_t *idx, uint32_
                                                     uint32_t *lnk) {
     static_assert((SLOTS & (SLOTS - 1)) == 0 && SLOTS >= 64 && SLOTS <= 65536, "slots: a power of two");
     constexpr uint32_t shift = 32u - static_cast<uint32_t>(__builtin_ctz(SLOTS));
-    __shared__ uint32_t key[D][SLOTS];
-    __shared__ uint16_t pos[D][SLOTS];
+    __shared__ uint32_t key[SLOTS];
+    __shared__ uint32_t val[SLOTS];
+    __shared__ uint32_t src[D];
     auto hash = [](uint32_t s) { return (s * 0x9E3779B1u) >> shift; };
     for (uint32_t j = blockIdx.x; j < n_sets; j += gridDim.x) {
-        for (uint32_t i = threadIdx.x; i < D * SLOTS; i += blockDim.x) (&key[0][0])[i] = kLinkEmpty;
+        for (uint32_t i = threadIdx.x; i < SLOTS; i += blockDim.x) {
+            key[i] = kLinkEmpty;
+            val[i] = 0xFFFFFFFFu;
+        }
+        if (threadIdx.x < D)
+            src[threadIdx.x] = static_cast<uint32_t>(
+                (static_cast<uint64_t>(j) + D * static_cast<uint64_t>(n_sets) - 1u - threadIdx.x) % n_sets);
         __syncthreads();
-        for (uint32_t t = 0; t < D; ++t) {
-            const uint32_t src =
-                static_cast<uint32_t>((static_cast<uint64_t>(j) + D * static_cast<uint64_t>(n_sets) - 1u - t) %
-                                      n_sets);
-            for (uint32_t m = threadIdx.x; m < K; m += blockDim.x) {
-                const uint32_t s = __ldg(idx + static_cast<size_t>(src) * K + m);
+        // D elements per thread at a time: their loads go out together, ahead
+        // of the table's atomics
+        for (uint32_t base = 0; base < D * K; base += D * blockDim.x) {
+            uint32_t sv[D], tv[D], mv[D];
+#pragma unroll
+            for (uint32_t i = 0; i < D; ++i) {
+                const uint32_t e = base + i * blockDim.x + threadIdx.x;
+                const bool in = e < D * K;
+                tv[i] = in ? e / K : 0u;
+                mv[i] = in ? e - tv[i] * K : 0u;
+                sv[i] = in ? __ldg(idx + static_cast<size_t>(src[tv[i]]) * K + mv[i]) : kLinkEmpty;
+            }
+#pragma unroll
+            for (uint32_t i = 0; i < D; ++i) {
+                const uint32_t s = sv[i];
                 if (s >= N) continue;
                 uint32_t h = hash(s);
                 for (uint32_t probe = 0; probe < SLOTS; ++probe) {
-                    const uint32_t prev = atomicCAS(&key[t][h], kLinkEmpty, s);
+                    const uint32_t prev = atomicCAS(&key[h], kLinkEmpty, s);
                     if (prev == kLinkEmpty || prev == s) {
-                        pos[t][h] = static_cast<uint16_t>(m);
+                        atomicMin(&val[h], ((tv[i] + 1u) << 16) | mv[i]);
                         break;
                     }
                     h = (h + 1u) & (SLOTS - 1u);
@@ -1615,17 +1633,15 @@ __global__ void __launch_bounds__(512) k_link_reach(const uint32_t *idx, uint32_
             const uint32_t s = __ldg(idx + static_cast<size_t>(j) * K + m);
             uint32_t l = 0;
             if (s < N) {
-                for (uint32_t t = 0; t < D && l == 0u; ++t) {
-                    uint32_t h = hash(s);
-                    for (uint32_t probe = 0; probe < SLOTS; ++probe) {
-                        const uint32_t k = key[t][h];
-                        if (k == s) {
-                            l = ((t + 1u) << 16) | pos[t][h];
-                            break;
-                        }
-                        if (k == kLinkEmpty) break;
-                        h = (h + 1u) & (SLOTS - 1u);
+                uint32_t h = hash(s);
+                for (uint32_t probe = 0; probe < SLOTS; ++probe) {
+                    const uint32_t k = key[h];
+                    if (k == s) {
+                        l = val[h];
+                        break;
                     }
+                    if (k == kLinkEmpty) break;
+                    h = (h + 1u) & (SLOTS - 1u);
                 }
             }
             lnk[static_cast<size_t>(j) * K + m] = l;
@@ -3625,12 +3641,12 @@ cudaError_t launch_link_pair(const StepArgs &a, uint32_t *lnk, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return e;
-    if (a.K > 256u) return cudaErrorInvalidValue;  // the tables hold 512 slots
+    if (a.K > 256u) return cudaErrorInvalidValue;  // the table holds 8 x 256 keys in 4,096 slots
     const uint32_t cap = static_cast<uint32_t>(sms) * 4u;
     const uint32_t grid = a.n_sets < cap ? a.n_sets : cap;
     const uint32_t threads = ((a.K + 31u) / 32u) * 32u;
-    k_link_reach<kPairD, 512><<<grid ? grid : 1u, threads ? threads : 32u, 0, s>>>(a.idx, a.n_sets, a.K,
-                                                                                   a.n_sessions, lnk);
+    k_link_reach<kPairD, 4096><<<grid ? grid : 1u, threads ? threads : 32u, 0, s>>>(a.idx, a.n_sets, a.K,
+                                                                                    a.n_sessions, lnk);
     return cudaGetLastError();
 }
 

@@ -310,7 +310,7 @@ def test_small_cohort_repeated_sessions(g, rc, monkeypatch, kernel, P, K, N):
     monkeypatch.setenv("RC_NO_PROD", "1" if kernel == "link" else "0")
     monkeypatch.setenv("RC_NO_PAIR", "0" if kernel == "pair" else "1")
     tables, state0, outc, pay, idx = _inputs(60 + K % 13 + P, K, 64, 16, P, 40, N=N)
-    n = 40
+    n = 70 if kernel == "pair" else 40  # the pair chain serves chains of 64 steps or more
     want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=1)
     got = g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K, sel0=1)
     g.assert_same(got, want, f"{kernel} K={K} N={N} P={P}")
@@ -358,7 +358,7 @@ def test_linked_single_cta_ring_wraps(g, rc, monkeypatch, SB, P, K, extra, want_
     S = 256 if SB == 64 else 64
     N = K + extra
     tables, state0, outc, pay, idx = _inputs(90 + n_sets + K % 7, K, S, SB, P, n_sets, N=N)
-    n = 13
+    n = 70 if kernel == "pair" else 13  # the pair chain serves chains of 64 steps or more
     want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=1)
     got = g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K, sel0=1)
     g.assert_same(got, want, f"linked n_sets={n_sets} SB={SB} P={P} K={K} N={N}")
