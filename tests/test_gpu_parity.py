@@ -185,6 +185,40 @@ def test_bad_inputs_are_latched_and_the_context_survives(g, rc):
     g.assert_same(g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K), want, "after errors")
 
 
+@pytest.mark.parametrize("what", ["outcome", "state", "index"])
+@pytest.mark.parametrize("K,identity", [(64, False), (256, False), (32, True)])
+def test_bad_inputs_in_two_step_chains(g, rc, what, K, identity):
+    """The chains that key two steps per block barrier (explicit sessions, 64
+    steps or more; identity sessions) latch a bad input with the step it sits
+    in and keep the context usable; a clean chain right after matches the
+    oracle."""
+    S, SB, P, n = 16, 16, 32, 70
+    tables, state0, outc, pay, idx = _inputs(150 + K, K, S, SB, P, n, N=None if identity else 4 * K)
+    if identity:
+        idx = None
+    st, oc, ix = state0.copy(), outc.copy(), None if idx is None else idx.copy()
+    bad_step, bad_member = 45, 5
+    if what == "outcome":
+        oc[bad_step, bad_member] = 8
+        code = rc.RC_E_STATE
+    elif what == "state":
+        sess = bad_member if identity else int(idx[0, bad_member])
+        st[sess, 0:4] = np.frombuffer(np.uint32(S).tobytes(), np.uint8)
+        bad_step, code = 0, rc.RC_E_STATE
+    else:
+        if identity:
+            pytest.skip("identity sessions have no index array")
+        ix[bad_step, bad_member] = 4 * K
+        code = rc.RC_E_INDEX
+    with pytest.raises(rc.RcError) as e:
+        g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, st, oc, pay, ix, n, K)
+    assert e.value.code == code
+    assert f"step {bad_step}," in str(e.value), str(e.value)
+    want = g.run_oracle(tables, state0, outc, pay, idx, n)
+    g.assert_same(g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K), want,
+                  f"after {what}")
+
+
 def test_grid_barrier_wait_is_bounded(g, rc, monkeypatch):
     """A CTA that never arrives (test hook) makes the others' bounded waits run
     out: RC_E_TIMEOUT comes back and the context keeps working."""
