@@ -646,9 +646,50 @@ def sweep(args):
         seg[str(R)] = {"one_segmented_launch_us_per_step": round(a, 3), "one_launch_per_route_us_per_step": round(b, 3),
                        "ratio": round(b / a, 3)}
 
+    # the replay cells: cohorts formed (deadline 50 ms, threshold K) from the
+    # arrivals of C active sessions, the first min(1,000, formed) of them per
+    # call, each mechanism; medians over repeated calls of the mean us per
+    # invocation, and the host round trip over the resident chain per cell
+    panel = wl.make_panel()
+    cells = {}
+    cell_mechs = {"resident_persist": rc.RC_MECH_RESIDENT_PERSIST, "host_rt": rc.RC_MECH_HOST_RT,
+                  "fixed_nested": rc.RC_MECH_FIXED_NESTED, "resident_cond": rc.RC_MECH_RESIDENT_COND}
+    for C in (10_000, 100_000):
+        arr = wl.make_arrivals(C, panel)
+        state0 = wl.make_state(arr.n_sessions, S, SB, wl.stream_seed(2, wl.Purpose.STATE))
+        ctab = wl.make_tables(S, wl.stream_seed(2, wl.Purpose.TABLE))
+        for K in (32, 64, 128, 256):
+            mem, _, _ = rc.form_cohorts(arr.t_ns, arr.route, arr.session, panel.n_labels, K, C2["delta_ns"])
+            n = min(1000, len(mem))
+            key = f"C={C},K={K}"
+            if n == 0:
+                cells[key] = {"formed_cohorts": 0, "note": "no qualifying cohort"}
+                continue
+            m_ = mem[:n]
+            outc = np.ascontiguousarray((arr.route[m_] % 8).astype(np.uint32))
+            idx = np.ascontiguousarray(arr.session[m_].astype(np.uint32))
+            pay = wl.payload_for_events(m_.reshape(-1), P).reshape(n, K, P)
+            ctx = rc.rc_init(S, ctab, SB, P, K, arr.n_sessions, stream)
+            dev_ev = (torch.from_numpy(outc.view(np.int32)).cuda(), torch.from_numpy(pay).cuda(),
+                      torch.from_numpy(idx.view(np.int32)).cuda())
+            state = torch.from_numpy(state0).cuda()
+            dec = torch.zeros(n, dtype=torch.int32, device="cuda")
+            res = {"formed_cohorts": int(len(mem)), "cohorts_per_call": n}
+            for name, mech in cell_mechs.items():
+                reps = 100 if name == "resident_persist" else 20
+                t = []
+                for r in range(reps + 2):
+                    ms, _ = chain_on_window(rc, ctx, mech, state, dev_ev, 0, n, K, dec, None)
+                    if r >= 2:
+                        t.append(ms * 1000.0 / n)
+                res[name] = round(float(np.median(t)), 4)
+            res["host_rt_over_resident"] = round(res["host_rt"] / res["resident_persist"], 3)
+            cells[key] = res
+            rc.rc_free(ctx)
+            del state, dev_ev, dec
+
     # the exact-packing grid of Section 5.2 on the GPU: C x seed swarms, three
     # groupings, deadlines x thresholds per swarm and grouping (540 rows)
-    panel = wl.make_panel()
     ks = [32, 64, 128, 256]
     ds = [10_000_000, 25_000_000, 50_000_000, 100_000_000, 250_000_000]
     grid_rows, gpu_s, gen_s, prop1 = 0, 0.0, 0.0, True
@@ -691,6 +732,9 @@ def sweep(args):
     return {"sweep": {"workload": "cohorts of N distinct sessions out of 4N, 16-byte state, 64-byte payload, "
                                   "S=64, ring of 64 cohorts; medians of repeated calls",
                       "opportunity_grid": opp_grid,
+                      "replay_cells": {"cells": cells, "unit": "us/invocation (median over calls)",
+                                       "mechanisms": list(cell_mechs),
+                                       "reps": "100 calls resident, 20 for the others"},
                       "segmented_routes_K256": seg,
                       "horizon_us_per_call": horizon, "ratio_host_rt_over_resident": ratio,
                       "safe_suffix": {"per_K_us_per_invocation": per_k, "K_r": k_r,
