@@ -646,6 +646,43 @@ def sweep(args):
         seg[str(R)] = {"one_segmented_launch_us_per_step": round(a, 3), "one_launch_per_route_us_per_step": round(b, 3),
                        "ratio": round(b / a, 3)}
 
+    # the long decision chain: K = 256 identity sessions, S = 128, A/B tables,
+    # 10,000 steps with the per-step log of states, effects and decisions,
+    # resident and host round trip timed; the two mechanisms' logs must agree
+    # element by element (their agreement with the oracle is tested on 50
+    # seeds in tests/test_gpu_workloads.py)
+    lc = wl.CONFIGS[5]
+    long_chain = {"seeds": [], "mismatches_resident_vs_host_rt": 0}
+    for seed in range(5):
+        cfg = 1000 + seed
+        Kl, Sl, nl, SBl, Pl = lc["K"], lc["S"], lc["n_steps"], lc["state_bytes"], lc["payload_bytes"]
+        ltab = wl.make_tables(Sl, wl.stream_seed(cfg, wl.Purpose.TABLE))
+        lstate0 = wl.make_state(Kl, Sl, SBl, wl.stream_seed(cfg, wl.Purpose.STATE))
+        lout, lpay, _ = wl.make_cohort_events(cfg, nl, Kl, Pl)
+        row, logs = {"seed": cfg}, {}
+        for name, mech in (("resident_persist", rc.RC_MECH_RESIDENT_PERSIST), ("host_rt", rc.RC_MECH_HOST_RT)):
+            ctx = rc.rc_init(Sl, ltab, SBl, Pl, Kl, Kl, stream)
+            lstate = torch.from_numpy(lstate0.copy()).cuda()
+            ev = rc.make_events(torch.from_numpy(lout.view(np.int32)).cuda(), torch.from_numpy(lpay).cuda(),
+                                None, payload_bytes=Pl, n_sets=nl)
+            dec = torch.zeros(nl, dtype=torch.int32, device="cuda")
+            eff = torch.zeros(nl * Kl * 16, dtype=torch.uint8, device="cuda")
+            slog = torch.zeros(nl * Kl * SBl, dtype=torch.uint8, device="cuda")
+            rc.rc_chain(ctx, nl, mech, lstate, ev, Kl, dec, eff, slog)
+            ms, _ = rc.rc_last_chain_stats(ctx)
+            logs[name] = [x.cpu().numpy() for x in (dec, eff, slog, lstate)]
+            row[name] = round(ms * 1000.0 / nl, 4)
+            rc.rc_free(ctx)
+            del lstate, dec, eff, slog
+        long_chain["mismatches_resident_vs_host_rt"] += sum(
+            int(np.count_nonzero(x != y)) for x, y in zip(logs["resident_persist"], logs["host_rt"]))
+        long_chain["seeds"].append(row)
+    long_chain["us_per_step_median"] = {
+        k: round(float(np.median([r[k] for r in long_chain["seeds"]])), 4) for k in ("resident_persist", "host_rt")}
+    long_chain["workload"] = ("long decision chain: K=256 identity sessions, S=128, 16-byte state, 32-byte payload, "
+                              "A/B tables, 10,000 steps, per-step logs on; seeds 1000..1004 (50 seeds against the "
+                              "oracle in the tests)")
+
     # the replay cells: cohorts formed (deadline 50 ms, threshold K) from the
     # arrivals of C active sessions, the first min(1,000, formed) of them per
     # call, each mechanism; medians over repeated calls of the mean us per
@@ -732,6 +769,7 @@ def sweep(args):
     return {"sweep": {"workload": "cohorts of N distinct sessions out of 4N, 16-byte state, 64-byte payload, "
                                   "S=64, ring of 64 cohorts; medians of repeated calls",
                       "opportunity_grid": opp_grid,
+                      "long_chain": long_chain,
                       "replay_cells": {"cells": cells, "unit": "us/invocation (median over calls)",
                                        "mechanisms": list(cell_mechs),
                                        "reps": "100 calls resident, 20 for the others"},
