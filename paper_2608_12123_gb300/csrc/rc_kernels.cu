@@ -79,6 +79,24 @@ __device__ __forceinline__ uint64_t route_key(uint32_t x, uint32_t o, const uint
     return h;
 }
 
+// Two independent route keys advanced round by round, so that the two
+// dependent chains interleave in the instruction stream.
+template <int P>
+__device__ __forceinline__ void route_key_pair(uint32_t xa, uint32_t oa, const uint4 (&pa)[P / 16], uint32_t xb,
+                                               uint32_t ob, const uint4 (&pb)[P / 16], uint64_t &ra, uint64_t &rb) {
+    uint64_t ha = fin64(pack64(xa, oa) ^ kGamma);
+    uint64_t hb = fin64(pack64(xb, ob) ^ kGamma);
+#pragma unroll
+    for (int k = 0; k < P / 16; ++k) {
+        ha = fin64(ha ^ pack64(pa[k].x, pa[k].y));
+        hb = fin64(hb ^ pack64(pb[k].x, pb[k].y));
+        ha = fin64(ha ^ pack64(pa[k].z, pa[k].w));
+        hb = fin64(hb ^ pack64(pb[k].z, pb[k].w));
+    }
+    ra = ha;
+    rb = hb;
+}
+
 // 64-bit word j (1..) of a record held as 16-byte vectors.
 template <int W, int NV>
 __device__ __forceinline__ uint64_t rec_word(const uint4 (&r)[NV]) {
@@ -594,9 +612,14 @@ __global__ void __launch_bounds__(512, 1) k_chain_cta_ident2(StepArgs a) {
 #pragma unroll
         for (int k = 0; k < NV; ++k) r[k] = rp[k];
     }
+    // event set of the next copy: advanced one step per call instead of a
+    // modulo (the copies go out in step order)
+    uint32_t next_set = 0;
     auto issue_data = [&](uint32_t j) {
+        const uint32_t set = next_set;
+        next_set = next_set + 1u == a.n_sets ? 0u : next_set + 1u;
         if (act && j < nst) {
-            const size_t e = static_cast<size_t>(j % a.n_sets) * K + m;
+            const size_t e = static_cast<size_t>(set) * K + m;
             cp_async4(&out_r[(j % RD) * Kp + m], a.outcome + e);
             const uint4 *src = reinterpret_cast<const uint4 *>(a.payload + e * P);
             uint4 *ring = pay_r + (j % RD) * Kp * NC;
@@ -639,6 +662,10 @@ __global__ void __launch_bounds__(512, 1) k_chain_cta_ident2(StepArgs a) {
         const uint32_t jb = ja + 1u;
         const bool has_b = jb < nst;
         cp_async_wait<D - 2>();  // this thread's data of steps ja and jb
+        // the copies of steps ja + D and ja + D + 1 (into the slots of steps
+        // ja - 2 and ja - 1, read last region) go out first
+        issue_data(ja + D);
+        issue_data(ja + D + 1u);
         if (pend) apply(ja - 1u, sel_b, pend_o, pend_rk);
         pend = false;
         uint32_t odd_a = 0, odd_b = 0;
@@ -664,8 +691,9 @@ __global__ void __launch_bounds__(512, 1) k_chain_cta_ident2(StepArgs a) {
                     pb[k] = ok_b ? rb[pay_chunk<P>(m, k)] : make_uint4(0, 0, 0, 0);
                 }
                 // two independent key chains (the second on a valid dummy when unused)
-                const uint64_t rk_a = route_key<P>(ok_a ? x_a : 0u, ok_a ? o_a : 0u, pa);
-                const uint64_t rk_b = route_key<P>(ok_b ? x_b : 0u, ok_b ? o_b : 0u, pb);
+                uint64_t rk_a, rk_b;
+                route_key_pair<P>(ok_a ? x_a : 0u, ok_a ? o_a : 0u, pa, ok_b ? x_b : 0u, ok_b ? o_b : 0u, pb, rk_a,
+                                  rk_b);
                 if (ok_a) {
                     apply(ja, sel_a, o_a, rk_a);
                     odd_a = static_cast<uint32_t>(rk_a & 1u);
@@ -678,8 +706,6 @@ __global__ void __launch_bounds__(512, 1) k_chain_cta_ident2(StepArgs a) {
                 }
             }
         }
-        issue_data(ja + D);
-        issue_data(ja + D + 1u);
         const uint32_t ca = __popc(__ballot_sync(0xffffffffu, odd_a != 0u));
         const uint32_t cb = __popc(__ballot_sync(0xffffffffu, odd_b != 0u));
         const uint32_t rr = (ja >> 1) & 1u;
@@ -689,6 +715,183 @@ __global__ void __launch_bounds__(512, 1) k_chain_cta_ident2(StepArgs a) {
         for (uint32_t w = 0; w < nw; ++w) total += warp_odd[rr][w];
         const uint32_t da = (total & 0xFFFFu) > K / 2u ? 1u : 0u;
         const uint32_t db = (total >> 16) > K / 2u ? 1u : 0u;
+        if (tid == 0 && a.decisions) {
+            a.decisions[ja] = da;
+            if (has_b) a.decisions[jb] = db;
+        }
+        sel_b = da;
+        sel_a = db;
+        last = has_b ? db : da;
+    }
+    if (pend) apply(nst - 1u, sel_b, pend_o, pend_rk);
+    cp_async_wait<0>();
+    if (act && in_range) {
+        uint4 *rp = reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(m) * SB);
+#pragma unroll
+        for (int k = 0; k < NV; ++k) rp[k] = r[k];
+    }
+    if (tid == 0) {
+        if (nst > 0) a.dev->sel = last;
+        a.dev->step = nst;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Persistent chain, one warp, member m = session m (K <= 32): the chain of
+// k_chain_cta_ident2 (two steps keyed side by side, the record of step 2r+1
+// updated at the next region's start) with the cohort inside one warp, so the
+// two counts of a region are the two ballots' popcounts and no block barrier
+// is needed; each lane reads only the ring slots its own copies fill.  Trace
+// points (lane 0, at step 2r): 0 region start, 1 data landed and copies
+// issued, 2 pending record updated, 3 second state ready, 4 keys done,
+// 5 record updated, 6 decisions.
+// ---------------------------------------------------------------------------
+template <int SB, int P, int D>
+__global__ void __launch_bounds__(32, 1) k_chain_warp_ident(StepArgs a) {
+    static_assert(D >= 2, "two steps per region");
+    constexpr uint32_t RD = D + 2;
+    constexpr uint32_t NC = P / 16;
+    constexpr int NV = SB / 16;
+    extern __shared__ __align__(16) uint8_t dsm[];
+    const uint32_t K = a.K;
+    const uint32_t Kp = (K + 3u) & ~3u;
+    const uint32_t tid = threadIdx.x;
+    uint8_t *tab = dsm;
+    uint32_t *out_r = reinterpret_cast<uint32_t *>(dsm + 2 * a.tab_stride);
+    uint4 *pay_r = reinterpret_cast<uint4 *>(out_r + RD * Kp);
+    stage_tables(tab, a.tables, a.tab_stride, 2, 0);
+    const bool act = tid < K;
+    const uint32_t m = tid;
+    const uint32_t nst = a.n_steps;
+    const bool in_range = m < a.n_sessions;
+    long long *trace = (a.trace && tid == 0) ? a.trace : nullptr;
+    uint4 r[NV];
+#pragma unroll
+    for (int k = 0; k < NV; ++k) r[k] = make_uint4(0, 0, 0, 0);
+    if (act && in_range) {
+        const uint4 *rp = reinterpret_cast<const uint4 *>(a.state + static_cast<size_t>(m) * SB);
+#pragma unroll
+        for (int k = 0; k < NV; ++k) r[k] = rp[k];
+    }
+    // event set of the next copy: advanced one step per call instead of a
+    // modulo (the copies go out in step order)
+    uint32_t next_set = 0;
+    auto issue_data = [&](uint32_t j) {
+        const uint32_t set = next_set;
+        next_set = next_set + 1u == a.n_sets ? 0u : next_set + 1u;
+        if (act && j < nst) {
+            const size_t e = static_cast<size_t>(set) * K + m;
+            cp_async4(&out_r[(j % RD) * Kp + m], a.outcome + e);
+            const uint4 *src = reinterpret_cast<const uint4 *>(a.payload + e * P);
+            uint4 *ring = pay_r + (j % RD) * Kp * NC;
+#pragma unroll
+            for (uint32_t k = 0; k < NC; ++k) cp_async16(ring + pay_chunk<P>(m, k), src + k);
+        }
+        cp_async_commit();
+    };
+    // this thread's record update for step n under decision sel (a valid member)
+    auto apply = [&](uint32_t n, uint32_t sel, uint32_t o, uint64_t rk) {
+        const uint32_t x = r[0].x;
+        const uint32_t y = tab[sel * a.tab_stride + x * 8u + o];
+        r[0].x = y;
+        r[0].y = r[0].y + 1u;
+        mix_acc<SB>(r, rk);
+        const size_t slot = static_cast<size_t>(n) * K + m;
+        if (a.effects) {
+            uint4 e;
+            e.x = static_cast<uint32_t>(rk);
+            e.y = static_cast<uint32_t>(rk >> 32);
+            e.z = m;
+            e.w = y | (o << 16) | (sel << 24);
+            __stcs(reinterpret_cast<uint4 *>(a.effects) + slot, e);
+        }
+        if (a.state_log) {
+            uint4 *lp = reinterpret_cast<uint4 *>(a.state_log + slot * SB);
+#pragma unroll
+            for (int k = 0; k < NV; ++k) __stcs(lp + k, r[k]);
+        }
+    };
+    for (uint32_t j = 0; j < D; ++j) issue_data(j);
+    __syncwarp();  // the tables staged by every lane
+    uint32_t sel_a = ld_volatile_u32(&a.dev->sel) & 1u;  // decision for step 2r: d(2r-1)
+    uint32_t sel_b = 0;                                  // decision for step 2r-1: d(2r-2)
+    bool pend = false;                                   // step 2r-1 keyed, record update pending
+    uint32_t pend_o = 0;
+    uint64_t pend_rk = 0;
+    uint32_t last = sel_a;  // the decision of the last step decided
+    for (uint32_t ja = 0; ja < nst; ja += 2u) {
+        const uint32_t jb = ja + 1u;
+        const bool has_b = jb < nst;
+        if (trace) trace[ja * 8 + 0] = clock64();
+        cp_async_wait<D - 2>();  // this thread's data of steps ja and jb
+        // the copies of steps ja + D and ja + D + 1 (into the slots of steps
+        // ja - 2 and ja - 1, read last region) go out first: their issue fills
+        // the stalls of the dependent lookups and keys below
+        issue_data(ja + D);
+        issue_data(ja + D + 1u);
+        if (trace) trace[ja * 8 + 1] = clock64();
+        if (pend) apply(ja - 1u, sel_b, pend_o, pend_rk);
+        pend = false;
+        if (trace) {
+            asm volatile("" ::"r"(r[0].x));
+            trace[ja * 8 + 2] = clock64();
+        }
+        uint32_t odd_a = 0, odd_b = 0;
+        if (act) {
+            const uint32_t o_a = out_r[(ja % RD) * Kp + m];
+            const uint32_t o_b = has_b ? out_r[(jb % RD) * Kp + m] : 0u;
+            if (!in_range) {
+                latch_error(a.dev, DEV_E_INDEX, ja, m);
+                if (has_b) latch_error(a.dev, DEV_E_INDEX, jb, m);
+            } else {
+                const uint32_t x_a = r[0].x;
+                const bool ok_a = x_a < a.S && o_a < 8u;
+                if (!ok_a) latch_error(a.dev, DEV_E_STATE, ja, m);
+                const uint32_t x_b = ok_a ? static_cast<uint32_t>(tab[sel_a * a.tab_stride + x_a * 8u + o_a]) : x_a;
+                const bool ok_b = has_b && x_b < a.S && o_b < 8u;
+                if (has_b && !ok_b) latch_error(a.dev, DEV_E_STATE, jb, m);
+                if (trace) {
+                    asm volatile("" ::"r"(x_b));
+                    trace[ja * 8 + 3] = clock64();
+                }
+                uint4 pa[NC], pb[NC];
+                const uint4 *ra = pay_r + (ja % RD) * Kp * NC;
+                const uint4 *rb = pay_r + (jb % RD) * Kp * NC;
+#pragma unroll
+                for (uint32_t k = 0; k < NC; ++k) {
+                    pa[k] = ra[pay_chunk<P>(m, k)];
+                    pb[k] = ok_b ? rb[pay_chunk<P>(m, k)] : make_uint4(0, 0, 0, 0);
+                }
+                // two independent key chains (the second on a valid dummy when unused)
+                uint64_t rk_a, rk_b;
+                route_key_pair<P>(ok_a ? x_a : 0u, ok_a ? o_a : 0u, pa, ok_b ? x_b : 0u, ok_b ? o_b : 0u, pb, rk_a,
+                                  rk_b);
+                if (trace) {
+                    asm volatile("" ::"l"(rk_a ^ rk_b));
+                    trace[ja * 8 + 4] = clock64();
+                }
+                if (ok_a) {
+                    apply(ja, sel_a, o_a, rk_a);
+                    odd_a = static_cast<uint32_t>(rk_a & 1u);
+                }
+                if (ok_b) {
+                    pend = true;
+                    pend_o = o_b;
+                    pend_rk = rk_b;
+                    odd_b = static_cast<uint32_t>(rk_b & 1u);
+                }
+            }
+        }
+        if (trace) trace[ja * 8 + 5] = clock64();
+        // the whole cohort is this warp: the counts are the ballots' own
+        const uint32_t ca = __popc(__ballot_sync(0xffffffffu, odd_a != 0u));
+        const uint32_t cb = __popc(__ballot_sync(0xffffffffu, odd_b != 0u));
+        const uint32_t da = ca > K / 2u ? 1u : 0u;
+        const uint32_t db = cb > K / 2u ? 1u : 0u;
+        if (trace) {
+            asm volatile("" ::"r"(da), "r"(db));
+            trace[ja * 8 + 6] = clock64();
+        }
         if (tid == 0 && a.decisions) {
             a.decisions[ja] = da;
             if (has_b) a.decisions[jb] = db;
@@ -3349,6 +3552,13 @@ const void *ident2_fn_rt(int SB, int P, int D) {
                       : reinterpret_cast<const void *>(&k_chain_cta_ident2<B, Q, 2>);
     });
 }
+const void *warp_fn_rt(int SB, int P, int D) {
+    return dispatch(SB, P, [&](auto b, auto q) {
+        constexpr int B = decltype(b)::value, Q = decltype(q)::value;
+        return D == 4 ? reinterpret_cast<const void *>(&k_chain_warp_ident<B, Q, 4>)
+                      : reinterpret_cast<const void *>(&k_chain_warp_ident<B, Q, 2>);
+    });
+}
 size_t ident2_smem(uint32_t K, int P, int D, uint32_t tab_stride) {
     const size_t Kp = (K + 3u) & ~3u, RD = D + 2;
     return 2 * tab_stride + RD * Kp * 4 + RD * Kp * P;
@@ -3369,6 +3579,18 @@ cudaError_t launch_chain_cta_fast(const StepArgs &a, int SB, int P, cudaStream_t
     const size_t cap = static_cast<size_t>(max_optin_smem());
     const uint32_t threads = ((K + 31u) / 32u) * 32u;
     StepArgs aa = a;
+    if (!a.idx && two_steps && K <= 32u) {
+        for (int D : {4, 2}) {
+            const size_t smem = ident2_smem(K, P, D, a.tab_stride);
+            if (smem > cap) continue;
+            const void *fn = warp_fn_rt(SB, P, D);
+            cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+            if (e != cudaSuccess) return e;
+            void *args[] = {&aa};
+            *launched = true;
+            return cudaLaunchKernel(fn, dim3(1), dim3(32), args, smem, s);
+        }
+    }
     if (!a.idx && two_steps && K <= 512u) {
         for (int D : {4, 2}) {
             const size_t smem = ident2_smem(K, P, D, a.tab_stride);
