@@ -86,8 +86,11 @@ typedef enum {
        handle and the flag in device memory selects the next route body. */
     RC_MECH_RESIDENT_COND = 1,
     /* Device resident, persistent kernel: one launch runs all steps; the
-       decision is reduced and read on device between steps (one CTA for
-       K <= 1024, a cooperative grid otherwise). */
+       decision is reduced and read on device between steps (one warp for
+       K <= 32 with identity sessions, one CTA for K <= 1024, one thread-block
+       cluster for K <= 8,192, a cooperative grid otherwise; the single-warp
+       and single-CTA forms key two consecutive steps per barrier where they
+       apply, which gives the same results). */
     RC_MECH_RESIDENT_PERSIST = 2,
     /* Fixed nested graph (Section 8.1 negative control): per step the host
        launches a graph whose launcher kernel device-launches a fixed child
@@ -190,10 +193,12 @@ int rc_launch_floor(rc_ctx *ctx, int kind, uint32_t reps, double *us_out);
 int rc_last_chain_stats(rc_ctx *ctx, double *device_ms_out, uint32_t *kernel_launches_out);
 
 /* Profiling aid: with a device buffer of at least 16 * n_steps int64 words
-   set, the persistent grid kernels record, for their first and last CTA, up
-   to eight SM clock readings (clock64) per step at their phase boundaries
-   (layout [2][n_steps][8]; the phases are listed beside each kernel in the
-   library source).  NULL (the default) turns it off. */
+   set, the persistent kernels that support it record up to eight SM clock
+   readings (clock64) per step at their phase boundaries: the grid kernels
+   for their first and last CTA (layout [2][n_steps][8]), the single-CTA and
+   single-warp ones for thread 0 (the first half; the two-step forms at their
+   even steps).  The phases are listed beside each kernel in the library
+   source.  NULL (the default) turns it off. */
 int rc_set_trace(rc_ctx *ctx, void *device_buf, uint64_t bytes);
 
 /* Test hook (device-side bounded-wait check): when armed, CTA 1 of the next
