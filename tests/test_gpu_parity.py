@@ -373,7 +373,8 @@ def test_single_cta_identity_sessions(g, rc, monkeypatch, mode, SB, P, K, n):
 @pytest.mark.parametrize("SB,P,K,extra,want_launches", [(16, 64, 256, 0, 2), (16, 64, 256, 1, 2), (16, 32, 7, 2, 2),
                                                    (64, 64, 256, 1, 2), (16, 128, 300, 3, 2), (64, 32, 33, 0, 2),
                                                    (16, 64, 264, 9, 2), (16, 64, 512, 5, 2), (64, 128, 512, 1, 1),
-                                                   (64, 128, 64, 3, 2), (16, 32, 8, 0, 2), (16, 128, 248, 40, 2)])
+                                                   (64, 128, 64, 3, 2), (16, 32, 8, 0, 2), (16, 128, 248, 40, 2),
+                                                   (64, 64, 64, 5, 2), (64, 32, 128, 9, 2), (64, 64, 128, 0, 2)])
 def test_linked_single_cta_ring_wraps(g, rc, monkeypatch, SB, P, K, extra, want_launches, n_sets, kernel):
     """The single-CTA chains that take recurring sessions from shared rings:
     cohorts drawn from N = K + extra sessions, so nearly every session recurs
