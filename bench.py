@@ -57,6 +57,8 @@ def parse_args():
     p.add_argument("--skip-large-k", action="store_true", help="omit the large-K bandwidth section")
     p.add_argument("--skip-cpu", action="store_true", help="omit the CPU-oracle baseline leg")
     p.add_argument("--large-k-only", action="store_true", help="run only the large-K section (profiling)")
+    p.add_argument("--tiny-only", action="store_true",
+                   help="run only the tiny chain's resident leg (profiling)")
     p.add_argument("--large-k-steps", type=int, default=1000)
     p.add_argument("--only-resident", action="store_true",
                    help="time only the resident chain of the headline workload (profiling)")
@@ -254,6 +256,9 @@ def native(args):
     stream = torch.cuda.current_stream()
     flush = None if args.no_flush else torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device="cuda")
 
+    if args.tiny_only:
+        print(json.dumps(tiny_chain(rc, torch, stream, mechanisms=("resident_persist",))))
+        return None
     if not args.large_k_only:
         w = make_config2()
         nc = w["n_cohorts"]
@@ -453,7 +458,7 @@ def large_k(args, rc, torch, stream, hbm_peak, peak_src, flush, world):
     }
 
 
-def tiny_chain(rc, torch, stream):
+def tiny_chain(rc, torch, stream, mechanisms=("resident_persist", "resident_cond", "host_rt")):
     """K = 32, S = 16, 16-byte records, 32-byte payloads, 1,000 chained steps,
     device-resident only: latency per step as a multiple of the launch floor."""
     c = wl.CONFIGS[1]
@@ -468,6 +473,8 @@ def tiny_chain(rc, torch, stream):
     out = {}
     for name, mech in (("resident_persist", rc.RC_MECH_RESIDENT_PERSIST), ("resident_cond", rc.RC_MECH_RESIDENT_COND),
                        ("host_rt", rc.RC_MECH_HOST_RT)):
+        if name not in mechanisms:
+            continue
         l = []
         for r in range(6):
             rc.rc_chain(ctx, n, mech, state, ev, K, dec, None, None)
