@@ -101,7 +101,7 @@ typedef enum {
        graph of step kernels without computing or reading any decision.  Not
        an admissible policy; a structural floor. */
     RC_MECH_FLOOR = 4,
-    /* The resident mechanism this build measured fastest for the shape
+    /* The resident mechanism measured fastest for the shape
        (currently the persistent kernel). */
     RC_MECH_RESIDENT = 5
 } rc_mechanism;

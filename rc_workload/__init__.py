@@ -317,7 +317,7 @@ def payload_for_events(event_ids: np.ndarray, payload_bytes: int, config_id: int
 
 
 # ----------------------------------------------------------------------------
-# The five workloads (shapes of the paper's studies at this build's sizes)
+# The five workloads (shapes of the paper's studies, at the sizes measured here)
 # ----------------------------------------------------------------------------
 
 CONFIGS = {
