@@ -196,8 +196,8 @@ int rc_last_chain_stats(rc_ctx *ctx, double *device_ms_out, uint32_t *kernel_lau
    set, the persistent kernels that support it record up to eight SM clock
    readings (clock64) per step at their phase boundaries: the grid kernels
    for their first and last CTA (layout [2][n_steps][8]), the single-CTA and
-   single-warp ones for thread 0 (the first half; the two-step forms at their
-   even steps).  The phases are listed beside each kernel in the library
+   single-warp ones for thread 0 (the first half); the two-step forms record
+   at their even steps.  The phases are listed beside each kernel in the library
    source.  NULL (the default) turns it off. */
 int rc_set_trace(rc_ctx *ctx, void *device_buf, uint64_t bytes);
 

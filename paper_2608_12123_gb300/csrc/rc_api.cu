@@ -98,6 +98,7 @@ struct rc_ctx {
     bool no_pair = false;   // RC_NO_PAIR=1 turns off the single-CTA chain keying two steps per barrier
     bool no_pieces = false; // RC_NO_PIECES=1 stages host-memory events whole (no pieces)
     bool no_grid_link = false;  // RC_NO_GRID_LINK=1 turns off the grid chain split by links
+    bool grid_pair = false;     // RC_GRID_PAIR=1 takes the grid chain keying two steps per barrier (measured slower)
     bool no_cluster = false;    // RC_NO_CLUSTER=1 turns off the cluster chain (512 < K <= 8192)
     bool use_split = false;  // RC_SPLIT=1 selects the split-phase chain (slower on GB300 so far)
     bool use_owned = false;  // RC_OWNED=1 selects the session-owned chain
@@ -491,6 +492,21 @@ int run_persist(rc_ctx *c, const rc::StepArgs &a) {
     if (!c->coop) return fail(c, RC_E_UNSUPPORTED, "device lacks cooperative launch");
     RC_CUDA(c, cudaMemsetAsync(c->dev->slot, 0, sizeof(c->dev->slot), c->stream));
     RC_CUDA(c, cudaMemsetAsync(&c->dev->abort, 0, sizeof(uint32_t), c->stream));
+    if (a.idx && c->grid_pair) {
+        int grid = 0;
+        uint32_t threads = 0;
+        size_t smem = 0, scratch = 0;
+        alignas(8) unsigned char shape[48];
+        if (rc::chain_grid_pair_plan(c->SB, c->P, a.K, c->n_sessions, a.n_sets, c->tab_stride, &grid, &threads, &smem,
+                                     shape, &scratch)) {
+            int rc = ensure(c, c->link_buf, scratch);
+            if (rc != RC_OK) return rc;
+            c->last_launches = 3;  // position and link passes, chain
+            RC_CUDA(c, rc::launch_chain_grid_pair(a, c->SB, c->P, grid, threads, smem, shape, c->link_buf.p, c->stream));
+            RC_CUDA(c, cudaMemsetAsync(&c->dev->skip_arrival, 0, sizeof(uint32_t), c->stream));
+            return RC_OK;
+        }
+    }
     if (a.idx && !c->no_grid_link) {
         int grid = 0;
         uint32_t threads = 0;
@@ -738,6 +754,8 @@ int rc_init(rc_ctx **out, uint32_t S, const uint8_t *table, uint32_t state_bytes
         c->no_pieces = np && np[0] == '1';
         const char *gl = std::getenv("RC_NO_GRID_LINK");
         c->no_grid_link = gl && gl[0] == '1';
+        const char *gp = std::getenv("RC_GRID_PAIR");
+        c->grid_pair = gp && gp[0] == '1';
         const char *cl = std::getenv("RC_NO_CLUSTER");
         c->no_cluster = cl && cl[0] == '1';
         const char *x = std::getenv("RC_SPLIT");

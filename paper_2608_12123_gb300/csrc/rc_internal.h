@@ -158,6 +158,17 @@ bool chain_grid_link_plan(int state_bytes, int payload_bytes, uint32_t K, uint64
 cudaError_t launch_chain_grid_link(const StepArgs &a, int state_bytes, int payload_bytes, int grid, uint32_t threads,
                                    size_t smem, const void *shape, void *scratch, cudaStream_t s);
 
+// Grid chain keying two steps per grid barrier (explicit indices, K a
+// multiple of 8 and at most 65,536): plan fills 48 bytes of opaque shape and
+// the scratch size (cohort bitmaps, per-cohort session positions, link
+// words, input-state and key rings); launch clears the bitmaps, runs the link
+// pass and the chain.
+bool chain_grid_pair_plan(int state_bytes, int payload_bytes, uint32_t K, uint64_t n_sessions, uint32_t n_sets,
+                          uint32_t tab_stride, int *grid, uint32_t *threads, size_t *smem, void *shape_out,
+                          size_t *scratch);
+cudaError_t launch_chain_grid_pair(const StepArgs &a, int state_bytes, int payload_bytes, int grid, uint32_t threads,
+                                   size_t smem, const void *shape, void *scratch, cudaStream_t s);
+
 // Split-phase persistent chain (explicit session indices, K a multiple of 8,
 // at most 512 members per CTA): marks is device scratch of 3 * n_sessions
 // words, filled with 0xFF bytes before each launch.

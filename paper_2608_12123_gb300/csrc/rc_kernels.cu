@@ -1945,8 +1945,9 @@ __global__ void __launch_bounds__(800, 1)
     uint8_t *const os = reinterpret_cast<uint8_t *>(xs + static_cast<size_t>(RX) * K);
     uint8_t *const fls = os + static_cast<size_t>(RX) * K;
     uint8_t *const tab = fls + static_cast<size_t>(RK) * K;
-    auto word_of = [&](uint32_t j, uint32_t which) { return words + (static_cast<size_t>(j % RW) * 3 + which) * K; };
-    auto rec_of = [&](uint32_t j, uint32_t q) { return rec + (static_cast<size_t>(j % RR) * K + q) * NV; };
+    // ring offsets stay below 2^20 elements: 32-bit arithmetic
+    auto word_of = [&](uint32_t j, uint32_t which) { return words + ((j % RW) * 3u + which) * K; };
+    auto rec_of = [&](uint32_t j, uint32_t q) { return rec + ((j % RR) * K + q) * NV; };
     const uint64_t stream_pol = policy_evict_first();
     long long *trace = (a.trace && tid == 0) ? a.trace : nullptr;
 
@@ -2573,6 +2574,506 @@ __global__ void __launch_bounds__(544, 1)
             for (uint32_t j = n; j < issued; ++j) (void)mbar_wait_bounded(&bar[j & 1u], (j >> 1) & 1u, limit);
         } else if (blockIdx.x == 0 && nst > 0) {
             a.dev->sel = sel;
+            a.dev->step = nst;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Persistent chain, cooperative grid, two steps per grid barrier (explicit
+// session indices, K a multiple of 8 and at most 65,536; one CTA per SM, CTA
+// b owns the members [b*chunk, b*chunk + cnt) of every step).
+//
+// The route key of step j needs the decisions only up to d(j - 2): the state
+// a session enters step j with is T_sel(i)[x_i][o_i] for its last step i < j,
+// and sel(i) = d(i - 1).  So region r, which starts once the barrier has
+// published d(2r - 2) and d(2r - 1), keys steps 2r and 2r + 1 together, and
+// its barrier publishes both odd counts; the records of those two steps are
+// completed (their transitions need d(2r - 1) and d(2r)) in region r + 1.
+//
+// The link pass (k_mark_pos, k_link_grid2) gives each member the nearest of
+// the three earlier cohorts holding its session (distance t, position q), a
+// forward bit (its session is in the next cohort) and, for t = 1, the same
+// link one level further back.  Every member writes its input state and
+// outcome to the ring `xo` (four steps) and, on even steps, its key to the
+// ring `keyring` (two even steps); other CTAs read them after the barrier.
+//  * x of an even step 2r: t in {1, 2} -> T_sel(i)[x_i][o_i] from xo, i =
+//    2r - t (keyed in region r - 1); otherwise the state array (the session's
+//    last step is at most 2r - 3, completed in region r - 1 at the latest).
+//  * x of an odd step 2r + 1: t in {2, 3} the same way; t = 1 (the session is
+//    in step 2r, keyed in this region by its owner) -> x of step 2r from the
+//    second link, then T_d(2r - 1)[x][outcome of step 2r]; otherwise the
+//    state array.
+//  * completing steps 2r - 2 and 2r - 1 in region r: a member of the even
+//    step whose session is in the odd one neither gathers nor stores: the
+//    odd step's member gathers the record, applies both steps (the first
+//    with the key from the ring) and stores once, writing both log rows.
+//    No other CTA touches that session's record in the region.
+// Region r, member threads: A1 gather the records of steps 2r - 2 and
+// 2r - 1 (warp-cooperatively), load x of steps 2r and 2r + 1 and the words
+// of steps 2r + 2 and 2r + 3; A3 complete, store and emit steps 2r - 2 and
+// 2r - 1; A2 wait for the payload tiles, key steps 2r and 2r + 1, write the
+// rings, count.  Then the control thread adds (1 << 48 | odd(2r + 1) << 24 |
+// odd(2r)) to the barrier word with release semantics, issues the payload
+// tiles of steps 2r + 3 and 2r + 4 (three tile stages) and spins.  Every
+// wait is bounded; a CTA that gives up latches RC_E_TIMEOUT, raises
+// dev->abort and leaves after the next block barrier, the control thread
+// first waiting (bounded) for its tile copies in flight.
+// ---------------------------------------------------------------------------
+struct GridPairShape {
+    TmaShape t;        // chunk, payload tiles, stage size (stage_words unused)
+    uint32_t members;  // member threads (a multiple of 32, >= chunk); the control warp follows
+    uint32_t pad[3];
+};
+constexpr uint32_t kGridPairStages = 3;  // payload tile stages
+constexpr uint32_t kGridPairThreads = 480;
+
+// bits[j] marks cohort j's sessions, pos[j][s] = the position of session s
+// in cohort j (read only where the bit is set; the caller clears the bits).
+__global__ void k_mark_pos(const uint32_t *idx, uint32_t n_sets, uint32_t K, uint64_t N, uint64_t words_per_set,
+                           uint32_t *bits, uint16_t *pos) {
+    const size_t total = static_cast<size_t>(n_sets) * K;
+    for (size_t e = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < total;
+         e += static_cast<size_t>(gridDim.x) * blockDim.x) {
+        const uint32_t s = idx[e];
+        if (s >= N) continue;
+        const size_t j = e / K;
+        atomicOr(bits + j * words_per_set + (s >> 5), 1u << (s & 31u));
+        pos[j * N + s] = static_cast<uint16_t>(e - j * K);
+    }
+}
+
+// lnk2[j][m] = {a, b}: a = fwd << 31 | t << 16 | q, the nearest cohort j - t
+// (t = 1..3, mod n_sets) holding member m's session at position q (t = 0:
+// none), fwd = the session is in cohort j + 1; for t = 1, b = t' << 16 | q',
+// the nearest of cohorts j - 2, j - 3 holding it, t' counted from j - 1.
+__global__ void k_link_grid2(const uint32_t *idx, uint32_t n_sets, uint32_t K, uint64_t N, uint64_t words_per_set,
+                             const uint32_t *bits, const uint16_t *pos, uint2 *lnk2) {
+    const size_t total = static_cast<size_t>(n_sets) * K;
+    for (size_t e = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < total;
+         e += static_cast<size_t>(gridDim.x) * blockDim.x) {
+        const uint32_t s = idx[e];
+        const uint64_t j = e / K;
+        uint2 w = make_uint2(0u, 0u);
+        if (s < N) {
+            auto back = [&](uint32_t t) { return (j + 3ull * n_sets - t) % n_sets; };
+            auto has = [&](uint64_t jj) { return ((bits[jj * words_per_set + (s >> 5)] >> (s & 31u)) & 1u) != 0u; };
+            auto at = [&](uint64_t jj) { return static_cast<uint32_t>(pos[jj * N + s]); };
+            for (uint32_t t = 1; t <= 3u; ++t) {
+                if (has(back(t))) {
+                    w.x = (t << 16) | at(back(t));
+                    break;
+                }
+            }
+            if (((w.x >> 16) & 3u) == 1u) {
+                for (uint32_t t = 2; t <= 3u; ++t) {
+                    if (has(back(t))) {
+                        w.y = ((t - 1u) << 16) | at(back(t));
+                        break;
+                    }
+                }
+            }
+            if (has((j + 1u) % n_sets)) w.x |= 1u << 31;
+        }
+        lnk2[e] = w;
+    }
+}
+
+template <int SB, int P>
+__global__ void __launch_bounds__(kGridPairThreads, 1)
+    k_chain_grid_pair(const __grid_constant__ CUtensorMap tmap, StepArgs a, const uint2 *lnk, uint32_t *xo,
+                      unsigned long long *keyring, GridPairShape gs) {
+    constexpr uint32_t NV = SB / 16;
+    constexpr uint32_t RPI = 32u / NV;
+    constexpr uint32_t NS = kGridPairStages;
+    constexpr uint32_t kSkip = 0, kRejected = 1, kApplied = 2;
+    const TmaShape sh = gs.t;
+    extern __shared__ uint8_t dsm_raw[];
+    __shared__ __align__(8) uint64_t pbar[NS];
+    __shared__ uint32_t warp_odd[2][16];
+    __shared__ uint32_t s_dec[4];  // d(i) at i & 3
+    __shared__ uint32_t s_sel0;
+    __shared__ uint32_t s_ab[2];  // [0]: raised before S1, read after it; [1]: raised in the spin, read after S2
+    // layout: [payload stage 0 | 1 | 2][records of the two completed steps][tables]
+    const uint32_t raw = smem_addr(dsm_raw);
+    uint8_t *const base = dsm_raw + (((raw + 1023u) & ~1023u) - raw);
+    uint4 *const recs = reinterpret_cast<uint4 *>(base + NS * sh.stage_pay);
+    uint8_t *const tab = reinterpret_cast<uint8_t *>(recs + 2ull * sh.chunk * NV);
+    auto pay_of = [&](uint32_t j) { return base + (j % NS) * sh.stage_pay; };
+    auto rec_of = [&](uint32_t i) { return recs + static_cast<size_t>(i) * sh.chunk * NV; };
+
+    const uint32_t tid = threadIdx.x;
+    const bool ctl = tid == gs.members;
+    const bool member = tid < gs.members;
+    const uint32_t lane = tid & 31u, wbase = tid & ~31u;
+    const uint32_t G = gridDim.x;
+    const uint32_t K = a.K;
+    const uint32_t m0 = blockIdx.x * sh.chunk;
+    const uint32_t cnt = m0 < K ? min(sh.chunk, K - m0) : 0u;
+    const bool mine = tid < cnt;  // this thread owns member p of every step
+    const uint32_t p = m0 + tid;
+    const uint32_t nst = a.n_steps;
+    const uint32_t S = a.S, stride = a.tab_stride;
+    const uint64_t N = a.n_sessions;
+    const uint64_t limit = a.dev->wait_ns;
+    const uint64_t stream_pol = policy_evict_first();
+    const uint64_t keep_pol = policy_evict_last();
+    long long *trace = nullptr;
+    if (a.trace && (tid == 0 || ctl) && (blockIdx.x == 0 || blockIdx.x == G - 1))
+        trace = a.trace + (blockIdx.x == 0 ? 0 : static_cast<size_t>(nst) * 8) + (ctl ? 0 : 4);
+
+    uint32_t issued = 0;  // control thread: the tiles of steps [0, issued) have been issued
+    auto issue = [&](uint32_t j) {
+        if (j >= nst || cnt == 0u) return;
+        issued = j + 1u;
+        uint64_t *b = &pbar[j % NS];
+        const uint32_t row0 = (j % a.n_sets) * K + m0;
+        mbar_arrive_expect_tx(b, sh.n_boxes * sh.box_rows * P);
+        for (uint32_t k = 0; k < sh.n_boxes; ++k)
+            tma_load_2d_hint(pay_of(j) + k * sh.box_rows * P, &tmap, 0, static_cast<int32_t>(row0 + k * sh.box_rows),
+                             b, stream_pol);
+    };
+    // the route body of step j: d(j - 1), d(-1) being the flag the chain starts from
+    auto sel_of = [&](uint32_t j) -> uint32_t { return j == 0u ? s_sel0 : s_dec[(j - 1u) & 3u]; };
+    auto body = [&](uint32_t j, uint32_t x, uint32_t o) -> uint32_t {
+        return (x < S && o < 8u) ? static_cast<uint32_t>(tab[sel_of(j) * stride + x * 8u + o]) : x;
+    };
+
+    if (ctl) {
+        for (uint32_t i = 0; i < NS; ++i) mbar_init(&pbar[i], 1);
+        fence_mbar_init();
+        s_sel0 = ld_volatile_u32(&a.dev->sel) & 1u;
+        for (uint32_t i = 0; i < 4u; ++i) s_dec[i] = 0;
+        s_ab[0] = 0;
+        s_ab[1] = 0;
+        for (uint32_t j = 0; j < NS; ++j) issue(j);
+    }
+    stage_tables(tab, a.tables, stride, 2, 0);
+
+    // words of this region's key steps (c*) and of the next region's (n*)
+    uint32_t co0 = 0, co1 = 0, cs0 = 0, cs1 = 0;
+    uint2 cl0 = make_uint2(0u, 0u), cl1 = make_uint2(0u, 0u);
+    uint32_t no0 = 0, no1 = 0, ns0 = 0, ns1 = 0;
+    uint2 nl0 = make_uint2(0u, 0u), nl1 = make_uint2(0u, 0u);
+    auto load_words = [&](uint32_t j, uint32_t &o, uint32_t &s, uint2 &l) {
+        if (mine && j < nst) {
+            const size_t e = static_cast<size_t>(j % a.n_sets) * K + p;
+            o = __ldcs(a.outcome + e);
+            s = __ldcs(a.idx + e);
+            l = __ldcs(lnk + e);
+        }
+    };
+    if (member) {
+        load_words(0, co0, cs0, cl0);
+        load_words(1, co1, cs1, cl1);
+    }
+    // carried from the key steps to their completion a region later
+    uint32_t ks0 = 0, ks1 = 0, ko0 = 0, ko1 = 0, kx0 = 0, kx1 = 0, kf0 = kSkip, kf1 = kSkip, kl0 = 0, kl1 = 0;
+    uint64_t krk0 = 0, krk1 = 0;
+    __syncthreads();
+
+    const uint32_t R = (nst + 1u) / 2u;  // key regions; region R only completes
+    uint32_t r = 0;
+    for (; r <= R; ++r) {
+        const uint32_t k0 = 2u * r, k1 = k0 + 1u;
+        const bool has_keys = k0 < nst;
+        long long *const tr = has_keys ? trace : nullptr;
+        if (member) {
+            if (tr) tr[k0 * 8 + 0] = clock64();
+            // ---- A1: gathers of the completed steps, loads of the key steps' x ----
+            const uint32_t c0 = k0 - 2u, c1 = k0 - 1u;  // valid when r > 0 (and < nst)
+            const bool done0 = r > 0 && c0 < nst, done1 = r > 0 && c1 < nst;
+            const bool fwd0 = (kl0 >> 31) != 0u && done1;     // the session goes on in step c1
+            const bool need0 = done0 && kf0 == kApplied && !fwd0;
+            const bool lnk1 = done1 && ((kl1 >> 16) & 3u) == 1u;  // in step c0 at position q1
+            const bool need1 = done1 && kf1 != kSkip && (kf1 == kApplied || lnk1);
+            uint64_t keyq = 0;
+            uint32_t oq = 8;
+            if (mine && need1 && lnk1) {
+                const uint32_t q1 = kl1 & 0xFFFFu;
+                keyq = __ldcg(keyring + static_cast<size_t>((c0 >> 1) & 1u) * K + q1);
+                oq = min(__ldg(a.outcome + static_cast<size_t>(c0 % a.n_sets) * K + q1), 8u);
+            }
+            {
+                const uint32_t c = lane % NV;
+                const uint32_t m_need0 = __ballot_sync(0xffffffffu, mine && need0);
+                const uint32_t m_need1 = __ballot_sync(0xffffffffu, mine && need1);
+#pragma unroll
+                for (uint32_t k = 0; k < NV; ++k) {
+                    const uint32_t q = k * RPI + lane / NV;
+                    const uint32_t s0 = __shfl_sync(0xffffffffu, ks0, q);
+                    const uint32_t s1 = __shfl_sync(0xffffffffu, ks1, q);
+                    if ((m_need0 >> q) & 1u)
+                        cp_async16(rec_of(0) + pay_chunk<SB>(wbase + q, c),
+                                   reinterpret_cast<const uint4 *>(a.state + static_cast<size_t>(s0) * SB) + c);
+                    if ((m_need1 >> q) & 1u)
+                        cp_async16(rec_of(1) + pay_chunk<SB>(wbase + q, c),
+                                   reinterpret_cast<const uint4 *>(a.state + static_cast<size_t>(s1) * SB) + c);
+                }
+                cp_async_commit();
+            }
+            // x sources of the key steps: a ring entry (packed x | o << 16,
+            // to pass through the body of its step) or the state array
+            const bool key0 = mine && has_keys, key1 = mine && k1 < nst;
+            const bool sv0 = key0 && cs0 < N, sv1 = key1 && cs1 < N;
+            uint32_t v0 = 0, v1 = 0, oe = 8, i0 = 0, i1 = 0;
+            bool ring0 = false, ring1 = false, chase1 = false;
+            if (sv0) {
+                const uint32_t t = (cl0.x >> 16) & 3u, q = cl0.x & 0xFFFFu;
+                if (t >= 1u && t <= 2u && t <= k0) {
+                    ring0 = true;
+                    i0 = k0 - t;
+                    v0 = __ldcg(xo + static_cast<size_t>(i0 & 3u) * K + q);
+                } else {
+                    v0 = __ldcg(reinterpret_cast<const uint32_t *>(a.state + static_cast<size_t>(cs0) * SB));
+                }
+            }
+            if (sv1) {
+                const uint32_t t = (cl1.x >> 16) & 3u, q = cl1.x & 0xFFFFu;
+                if (t == 1u) {
+                    chase1 = true;  // x of step k0 for this session, then step k0's body
+                    oe = min(__ldg(a.outcome + static_cast<size_t>(k0 % a.n_sets) * K + q), 8u);
+                    const uint32_t t2 = (cl1.y >> 16) & 3u, q2 = cl1.y & 0xFFFFu;
+                    if (t2 >= 1u && t2 <= 2u && t2 <= k0) {
+                        ring1 = true;
+                        i1 = k0 - t2;
+                        v1 = __ldcg(xo + static_cast<size_t>(i1 & 3u) * K + q2);
+                    } else {
+                        v1 = __ldcg(reinterpret_cast<const uint32_t *>(a.state + static_cast<size_t>(cs1) * SB));
+                    }
+                } else if (t >= 2u && t <= k1) {
+                    ring1 = true;
+                    i1 = k1 - t;
+                    v1 = __ldcg(xo + static_cast<size_t>(i1 & 3u) * K + q);
+                } else {
+                    v1 = __ldcg(reinterpret_cast<const uint32_t *>(a.state + static_cast<size_t>(cs1) * SB));
+                }
+            }
+            load_words(k0 + 2u, no0, ns0, nl0);
+            load_words(k1 + 2u, no1, ns1, nl1);
+            if (tr) tr[k0 * 8 + 1] = clock64();
+
+            // ---- A3: complete, store and emit steps c0 and c1 ----
+            cp_async_wait<0>();
+            __syncwarp();
+            bool st0 = false, st1 = false;
+            if (mine && done0 && kf0 == kApplied) {
+                const uint32_t sel = sel_of(c0);
+                const uint32_t y = tab[sel * stride + kx0 * 8u + ko0];
+                if (need0) {
+                    uint4 rr[NV];
+#pragma unroll
+                    for (uint32_t k = 0; k < NV; ++k) rr[k] = rec_of(0)[pay_chunk<SB>(tid, k)];
+                    rr[0].x = y;
+                    rr[0].y = rr[0].y + 1u;
+                    mix_acc<SB>(rr, krk0);
+#pragma unroll
+                    for (uint32_t k = 0; k < NV; ++k) rec_of(0)[pay_chunk<SB>(tid, k)] = rr[k];
+                    if (a.state_log) {
+                        uint4 *lp = reinterpret_cast<uint4 *>(a.state_log + (static_cast<size_t>(c0) * K + p) * SB);
+#pragma unroll
+                        for (uint32_t k = 0; k < NV; ++k) __stcs(lp + k, rr[k]);
+                    }
+                    st0 = true;
+                }
+                if (a.effects) {
+                    uint4 e;
+                    e.x = static_cast<uint32_t>(krk0);
+                    e.y = static_cast<uint32_t>(krk0 >> 32);
+                    e.z = ks0;
+                    e.w = y | (ko0 << 16) | (sel << 24);
+                    __stcs(reinterpret_cast<uint4 *>(a.effects) + static_cast<size_t>(c0) * K + p, e);
+                }
+            }
+            if (mine && need1) {
+                uint4 rr[NV];
+#pragma unroll
+                for (uint32_t k = 0; k < NV; ++k) rr[k] = rec_of(1)[pay_chunk<SB>(tid, k)];
+                if (lnk1 && rr[0].x < S && oq < 8u) {
+                    // step c0 of this session, whose member left the record to this one
+                    rr[0].x = tab[sel_of(c0) * stride + rr[0].x * 8u + oq];
+                    rr[0].y = rr[0].y + 1u;
+                    mix_acc<SB>(rr, keyq);
+                    if (a.state_log) {
+                        uint4 *lp = reinterpret_cast<uint4 *>(a.state_log +
+                                                              (static_cast<size_t>(c0) * K + (kl1 & 0xFFFFu)) * SB);
+#pragma unroll
+                        for (uint32_t k = 0; k < NV; ++k) __stcs(lp + k, rr[k]);
+                    }
+                    st1 = true;
+                }
+                if (kf1 == kApplied) {
+                    const uint32_t sel = sel_of(c1);
+                    const uint32_t y = tab[sel * stride + kx1 * 8u + ko1];
+                    rr[0].x = y;
+                    rr[0].y = rr[0].y + 1u;
+                    mix_acc<SB>(rr, krk1);
+                    if (a.state_log) {
+                        uint4 *lp = reinterpret_cast<uint4 *>(a.state_log + (static_cast<size_t>(c1) * K + p) * SB);
+#pragma unroll
+                        for (uint32_t k = 0; k < NV; ++k) __stcs(lp + k, rr[k]);
+                    }
+                    if (a.effects) {
+                        uint4 e;
+                        e.x = static_cast<uint32_t>(krk1);
+                        e.y = static_cast<uint32_t>(krk1 >> 32);
+                        e.z = ks1;
+                        e.w = y | (ko1 << 16) | (sel << 24);
+                        __stcs(reinterpret_cast<uint4 *>(a.effects) + static_cast<size_t>(c1) * K + p, e);
+                    }
+                    st1 = true;
+                }
+                if (st1) {
+#pragma unroll
+                    for (uint32_t k = 0; k < NV; ++k) rec_of(1)[pay_chunk<SB>(tid, k)] = rr[k];
+                }
+            }
+            {
+                const uint32_t m_st0 = __ballot_sync(0xffffffffu, st0);
+                const uint32_t m_st1 = __ballot_sync(0xffffffffu, st1);
+                __syncwarp();
+                const uint32_t c = lane % NV;
+#pragma unroll
+                for (uint32_t k = 0; k < NV; ++k) {
+                    const uint32_t q = k * RPI + lane / NV;
+                    const uint32_t s0 = __shfl_sync(0xffffffffu, ks0, q);
+                    const uint32_t s1 = __shfl_sync(0xffffffffu, ks1, q);
+                    if ((m_st0 >> q) & 1u)
+                        st_hint(reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(s0) * SB) + c,
+                                rec_of(0)[pay_chunk<SB>(wbase + q, c)], keep_pol);
+                    if ((m_st1 >> q) & 1u)
+                        st_hint(reinterpret_cast<uint4 *>(a.state + static_cast<size_t>(s1) * SB) + c,
+                                rec_of(1)[pay_chunk<SB>(wbase + q, c)], keep_pol);
+                }
+            }
+            if (tr) tr[k0 * 8 + 2] = clock64();
+
+            // ---- A2: key steps k0 and k1 ----
+            uint32_t odd0 = 0, odd1 = 0;
+            if (has_keys && cnt > 0u) {
+                bool landed = mbar_wait_bounded(&pbar[k0 % NS], (k0 / NS) & 1u, limit);
+                if (k1 < nst) landed = landed && mbar_wait_bounded(&pbar[k1 % NS], (k1 / NS) & 1u, limit);
+                if (!landed) {
+                    if (tid == 0) latch_error(a.dev, DEV_E_TIMEOUT, k0, blockIdx.x);
+                    s_ab[0] = 1;
+                } else {
+                    const uint32_t x0 = ring0 ? body(i0, v0 & 0xFFFFu, v0 >> 16) : v0;
+                    uint32_t x1 = ring1 ? body(i1, v1 & 0xFFFFu, v1 >> 16) : v1;
+                    // a bad state carried from step k0 is latched by that step's member
+                    const bool inherited = chase1 && x1 >= S;
+                    if (chase1) x1 = body(k0, x1, oe);
+                    const bool ok0 = sv0 && x0 < S && co0 < 8u, ok1 = sv1 && x1 < S && co1 < 8u;
+                    if (key0 && !ok0) latch_error(a.dev, sv0 ? DEV_E_STATE : DEV_E_INDEX, k0, p);
+                    if (key1 && !ok1 && !inherited) latch_error(a.dev, sv1 ? DEV_E_STATE : DEV_E_INDEX, k1, p);
+                    uint4 pa[P / 16], pb[P / 16];
+                    if (key0) {
+                        read_payload_swizzled<P>(pa, pay_of(k0), tid);
+                    } else {
+#pragma unroll
+                        for (int k = 0; k < P / 16; ++k) pa[k] = make_uint4(0u, 0u, 0u, 0u);
+                    }
+                    if (key1) {
+                        read_payload_swizzled<P>(pb, pay_of(k1), tid);
+                    } else {
+#pragma unroll
+                        for (int k = 0; k < P / 16; ++k) pb[k] = make_uint4(0u, 0u, 0u, 0u);
+                    }
+                    uint64_t rk0 = 0, rk1 = 0;
+                    route_key_pair<P>(ok0 ? x0 : 0u, ok0 ? co0 : 0u, pa, ok1 ? x1 : 0u, ok1 ? co1 : 0u, pb, rk0, rk1);
+                    odd0 = ok0 ? static_cast<uint32_t>(rk0 & 1u) : 0u;
+                    odd1 = ok1 ? static_cast<uint32_t>(rk1 & 1u) : 0u;
+                    if (key0) {
+                        __stcg(xo + static_cast<size_t>(k0 & 3u) * K + p, min(x0, 0xFFFFu) | (min(co0, 8u) << 16));
+                        __stcg(keyring + static_cast<size_t>((k0 >> 1) & 1u) * K + p,
+                               static_cast<unsigned long long>(rk0));
+                    }
+                    if (key1) __stcg(xo + static_cast<size_t>(k1 & 3u) * K + p, min(x1, 0xFFFFu) | (min(co1, 8u) << 16));
+                    ks0 = cs0;
+                    ko0 = co0;
+                    kx0 = x0;
+                    krk0 = rk0;
+                    kl0 = cl0.x;
+                    kf0 = !key0 ? kSkip : (!sv0 ? kSkip : (ok0 ? kApplied : kRejected));
+                    ks1 = cs1;
+                    ko1 = co1;
+                    kx1 = x1;
+                    krk1 = rk1;
+                    kl1 = cl1.x;
+                    kf1 = !key1 ? kSkip : (!sv1 ? kSkip : (ok1 ? kApplied : kRejected));
+                }
+            }
+            const uint32_t w = tid >> 5;
+            const uint32_t n0 = __popc(__ballot_sync(0xffffffffu, odd0 != 0u));
+            const uint32_t n1 = __popc(__ballot_sync(0xffffffffu, odd1 != 0u));
+            if (lane == 0) {
+                warp_odd[0][w] = n0;
+                warp_odd[1][w] = n1;
+            }
+            co0 = no0;
+            cs0 = ns0;
+            cl0 = nl0;
+            co1 = no1;
+            cs1 = ns1;
+            cl1 = nl1;
+            if (tr) tr[k0 * 8 + 3] = clock64();
+        }
+        __syncthreads();  // S1: records stored, rings written, counts staged, tiles read
+        if (s_ab[0] != 0u || !has_keys) break;
+        if (ctl) {
+            if (tr) tr[k0 * 8 + 0] = clock64();
+            uint32_t ce = 0, cd = 0;
+            for (uint32_t w = 0; w < gs.members / 32u; ++w) {
+                ce += warp_odd[0][w];
+                cd += warp_odd[1][w];
+            }
+            unsigned long long *word = &a.dev->slot[r % 3u];
+            if (blockIdx.x == 0) a.dev->slot[(r + 1u) % 3u] = 0ull;
+            const bool skip = (r == 0 && blockIdx.x == 1 && ld_volatile_u32(&a.dev->skip_arrival) != 0u);
+            if (!skip) red_release_add_u64(word, (1ull << 48) | (static_cast<unsigned long long>(cd) << 24) | ce);
+            if (tr) tr[k0 * 8 + 1] = clock64();
+            fence_proxy_async_smem();
+            issue(k0 + 3u);
+            issue(k1 + 3u);
+            if (tr) tr[k0 * 8 + 2] = clock64();
+            uint64_t t0 = 0;
+            unsigned long long wv;
+            uint32_t spins = 0;
+            for (;;) {
+                wv = ld_acquire_u64(word);
+                if ((wv >> 48) >= G) break;
+                if ((++spins & 63u) == 0u) {
+                    if (ld_volatile_u32(&a.dev->abort) != 0u) {
+                        s_ab[1] = 1;
+                        break;
+                    }
+                    if (timed_out(t0, limit)) {
+                        latch_error(a.dev, DEV_E_TIMEOUT, k0, blockIdx.x);
+                        atomicExch(&a.dev->abort, 1u);
+                        s_ab[1] = 1;
+                        break;
+                    }
+                }
+            }
+            const uint32_t d0 = (static_cast<uint32_t>(wv & 0xFFFFFFull) > K / 2u) ? 1u : 0u;
+            const uint32_t d1 = (static_cast<uint32_t>((wv >> 24) & 0xFFFFFFull) > K / 2u) ? 1u : 0u;
+            s_dec[k0 & 3u] = d0;
+            s_dec[k1 & 3u] = d1;
+            if (blockIdx.x == 0 && a.decisions && s_ab[1] == 0u) {
+                a.decisions[k0] = d0;
+                if (k1 < nst) a.decisions[k1] = d1;
+            }
+            if (tr) tr[k0 * 8 + 3] = clock64();
+        }
+        __syncthreads();  // S2: d(k0), d(k1) known
+        if (s_ab[1] != 0u) break;
+    }
+    cp_async_wait<0>();
+    if (ctl) {
+        if (r < R) {
+            // stopped early: wait (bounded) for the tile copies still in flight
+            for (uint32_t j = 2u * r; j < issued; ++j) (void)mbar_wait_bounded(&pbar[j % NS], (j / NS) & 1u, limit);
+        } else if (blockIdx.x == 0 && nst > 0) {
+            a.dev->sel = sel_of(nst);
             a.dev->step = nst;
         }
     }
@@ -4012,6 +4513,106 @@ cudaError_t launch_chain_grid_link(const StepArgs &a, int SB, int P, int grid, u
     const uint32_t *l = lnk;
     void *args[] = {&map, &aa, &l, &gs};
     return cudaLaunchCooperativeKernel(grid_link_fn(SB, P), dim3(grid), dim3(threads), args, smem, s);
+}
+
+namespace {
+const void *grid_pair_fn(int SB, int P) {
+    return dispatch(SB, P, [](auto b, auto q) {
+        return reinterpret_cast<const void *>(&k_chain_grid_pair<decltype(b)::value, decltype(q)::value>);
+    });
+}
+// Byte offsets of the two-step grid chain's scratch: cohort bitmaps, session
+// positions per cohort, link words, the input-state ring and the key ring
+// (each part 256-byte aligned).
+struct GridPairScratch {
+    size_t pos, lnk, xo, keys, total;
+};
+GridPairScratch grid_pair_scratch(uint32_t K, uint64_t N, uint32_t n_sets) {
+    auto up = [](size_t v) { return (v + 255u) & ~static_cast<size_t>(255u); };
+    const uint64_t words_per_set = (N + 31u) / 32u;
+    GridPairScratch o{};
+    o.pos = up(static_cast<size_t>(n_sets) * words_per_set * 4);
+    o.lnk = o.pos + up(static_cast<size_t>(n_sets) * N * 2);
+    o.xo = o.lnk + up(static_cast<size_t>(n_sets) * K * 8);
+    o.keys = o.xo + up(4ull * K * 4);
+    o.total = o.keys + up(2ull * K * 8);
+    return o;
+}
+}  // namespace
+
+bool chain_grid_pair_plan(int SB, int P, uint32_t K, uint64_t n_sessions, uint32_t n_sets, uint32_t tab_stride,
+                          int *grid, uint32_t *threads, size_t *smem, void *shape_out, size_t *scratch) {
+    if (K == 0 || K % 8u != 0u || K > 65536u || n_sessions > 0xFFFFFFFFull || !encode_fn()) return false;
+    int dev = 0, sms = 0, max_optin = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return false;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return false;
+    if (cudaDeviceGetAttribute(&max_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+        return false;
+    GridPairShape gs{};
+    TmaShape &sh = gs.t;
+    const uint32_t per = (K + static_cast<uint32_t>(sms) - 1u) / static_cast<uint32_t>(sms);
+    sh.chunk = (per + 7u) & ~7u;
+    const uint32_t g = (K + sh.chunk - 1u) / sh.chunk;
+    sh.n_boxes = (sh.chunk + 255u) / 256u;
+    sh.box_rows = (((sh.chunk + sh.n_boxes - 1u) / sh.n_boxes) + 7u) & ~7u;
+    sh.stage_pay = ((sh.n_boxes * sh.box_rows * static_cast<uint32_t>(P)) + 1023u) & ~1023u;
+    sh.stage_words = 0;
+    gs.members = ((sh.chunk + 31u) / 32u) * 32u;
+    if (gs.members + 32u > kGridPairThreads) return false;
+    const size_t bytes = 1024 + static_cast<size_t>(kGridPairStages) * sh.stage_pay + 2ull * sh.chunk * SB +
+                         ((2ull * tab_stride + 15u) & ~15ull);
+    if (bytes > static_cast<size_t>(max_optin)) return false;
+    const GridPairScratch o = grid_pair_scratch(K, n_sessions, n_sets);
+    if (o.total > (1ull << 30)) return false;
+    const void *fn = grid_pair_fn(SB, P);
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes)) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, static_cast<int>(gs.members + 32u), bytes) !=
+            cudaSuccess ||
+        per_sm < 1 || static_cast<long long>(per_sm) * sms < g)
+        return false;
+    *grid = static_cast<int>(g);
+    *threads = gs.members + 32u;
+    *smem = bytes;
+    *scratch = o.total;
+    static_assert(sizeof(GridPairShape) <= 48, "shape buffer");
+    std::memcpy(shape_out, &gs, sizeof(gs));
+    return true;
+}
+
+cudaError_t launch_chain_grid_pair(const StepArgs &a, int SB, int P, int grid, uint32_t threads, size_t smem,
+                                   const void *shape, void *scratch, cudaStream_t s) {
+    GridPairShape gs;
+    std::memcpy(&gs, shape, sizeof(gs));
+    const GridPairScratch o = grid_pair_scratch(a.K, a.n_sessions, a.n_sets);
+    uint8_t *const base = static_cast<uint8_t *>(scratch);
+    uint32_t *bits = reinterpret_cast<uint32_t *>(base);
+    uint16_t *pos = reinterpret_cast<uint16_t *>(base + o.pos);
+    uint2 *lnk = reinterpret_cast<uint2 *>(base + o.lnk);
+    uint32_t *xo = reinterpret_cast<uint32_t *>(base + o.xo);
+    unsigned long long *keys = reinterpret_cast<unsigned long long *>(base + o.keys);
+    const uint64_t words_per_set = (a.n_sessions + 31u) / 32u;
+    cudaError_t e = cudaMemsetAsync(bits, 0, static_cast<size_t>(a.n_sets) * words_per_set * 4, s);
+    if (e != cudaSuccess) return e;
+    int dev = 0, sms = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+    const size_t total = static_cast<size_t>(a.n_sets) * a.K;
+    const size_t want = (total + 255u) / 256u;
+    const unsigned blocks = static_cast<unsigned>(want < static_cast<size_t>(sms) * 8u ? want : static_cast<size_t>(sms) * 8u);
+    k_mark_pos<<<blocks ? blocks : 1u, 256, 0, s>>>(a.idx, a.n_sets, a.K, a.n_sessions, words_per_set, bits, pos);
+    k_link_grid2<<<blocks ? blocks : 1u, 256, 0, s>>>(a.idx, a.n_sets, a.K, a.n_sessions, words_per_set, bits, pos,
+                                                      lnk);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    alignas(64) CUtensorMap map;
+    if (!payload_map(a, P, gs.t.box_rows, &map)) return cudaErrorInvalidValue;
+    StepArgs aa = a;
+    const uint2 *l = lnk;
+    void *args[] = {&map, &aa, &l, &xo, &keys, &gs};
+    return cudaLaunchCooperativeKernel(grid_pair_fn(SB, P), dim3(grid), dim3(threads), args, smem, s);
 }
 
 namespace {

@@ -259,24 +259,80 @@ def test_launch_floor_probes_run(g, rc):
         rc.rc_free(ctx)
 
 
+@pytest.mark.parametrize("kernel", ["gpair", "link"])
 @pytest.mark.parametrize("n_sets", [1, 2, 3, 4, 7])
 @pytest.mark.parametrize("SB,P,K,N", [(64, 128, 2056, 2100), (16, 64, 4104, 12000), (64, 32, 1032, 1032)])
-def test_grid_link_records_stored_early_and_late(g, rc, monkeypatch, n_sets, SB, P, K, N):
-    """The grid chain split by links over many steps: sessions recurring at
-    distances 1, 2, 3 and more (rings of 1 to 7 cohorts drawn from N near K)
-    must see every earlier record, whether it reaches them through the
-    linked gather after the barrier or the unlinked gather run ahead while the
-    barrier is awaited."""
+def test_grid_link_records_stored_early_and_late(g, rc, monkeypatch, kernel, n_sets, SB, P, K, N):
+    """The grid chains over many steps: sessions recurring at distances 1, 2,
+    3 and more (rings of 1 to 7 cohorts drawn from N near K) must see every
+    earlier record.  "link" (one step per barrier): through the linked gather
+    after the barrier or the unlinked gather run ahead while it is awaited;
+    "gpair" (two steps per barrier): through the input-state ring, the
+    second link of an odd step whose session is in the even one, the record
+    handed from the even step to the odd one, or the state array."""
     monkeypatch.setenv("RC_NO_CLUSTER", "1")
+    monkeypatch.setenv("RC_GRID_PAIR", "1" if kernel == "gpair" else "0")
     S = 256 if SB == 64 else 64
     tables, state0, outc, pay, idx = _inputs(140 + n_sets + K % 7, K, S, SB, P, n_sets, N=N)
     n = 14
     want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=1)
     got = g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K, sel0=1)
-    g.assert_same(got, want, f"grid link n_sets={n_sets} SB={SB} P={P} K={K} N={N}")
+    g.assert_same(got, want, f"grid {kernel} n_sets={n_sets} SB={SB} P={P} K={K} N={N}")
 
 
-@pytest.mark.parametrize("kernel", ["link", "owned", "split", "tma", "plain"])
+@pytest.mark.parametrize("n", [1, 2, 3, 4, 5, 13])
+@pytest.mark.parametrize("n_sets", [1, 2, 5])
+@pytest.mark.parametrize("SB,P", [(16, 32), (64, 128)])
+def test_grid_pair_step_counts(g, rc, monkeypatch, n, n_sets, SB, P):
+    """Two steps per grid barrier on chains of odd and even length, the
+    shortest among them (a region with one key step, a last region that only
+    completes), sessions recurring at every distance (N near K)."""
+    monkeypatch.setenv("RC_NO_CLUSTER", "1")
+    monkeypatch.setenv("RC_GRID_PAIR", "1")
+    K, N = 2056, 2300
+    S = 256 if SB == 64 else 64
+    tables, state0, outc, pay, idx = _inputs(170 + n + 7 * n_sets, K, S, SB, P, n_sets, N=N)
+    want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=n & 1)
+    got = g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K, sel0=n & 1)
+    g.assert_same(got, want, f"grid pair n={n} n_sets={n_sets} SB={SB} P={P}")
+
+
+@pytest.mark.parametrize("what", ["state_even", "state_odd", "outcome_even", "outcome_odd", "index_odd"])
+def test_grid_pair_errors_report_the_earlier_step(g, rc, monkeypatch, what):
+    """Two steps keyed in one region by different CTAs: a bad state first met
+    in the even step and carried into the odd one is reported at the even
+    step; a bad outcome or index is reported at its own step."""
+    monkeypatch.setenv("RC_NO_CLUSTER", "1")
+    monkeypatch.setenv("RC_GRID_PAIR", "1")
+    K, S, SB, P, n, N = 4104, 64, 16, 64, 6, 4400
+    tables, state0, outc, pay, idx = _inputs(190, K, S, SB, P, n, N=N)
+    st, oc, ix = state0.copy(), outc.copy(), idx.copy()
+    even = what.endswith("even")
+    if what.startswith("state"):
+        # the session's first step in the chain: step 0, its session also in
+        # step 1 (carried into the odd step); or step 1, its session not in 0
+        j = 0 if even else 1
+        pick = np.isin(idx[0], idx[1]) if even else ~np.isin(idx[1], idx[0])
+        m = int(np.flatnonzero(pick)[0])
+        st[int(idx[j, m]), 0:4] = np.frombuffer(np.uint32(S + 3).tobytes(), np.uint8)
+        code = rc.RC_E_STATE
+    else:
+        # step 2 with its session also in step 3, or step 3 with it in step 2
+        j = 2 if even else 3
+        m = int(np.flatnonzero(np.isin(idx[j], idx[j + 1] if even else idx[j - 1]))[0])
+        if what.startswith("outcome"):
+            oc[j, m] = 9
+            code = rc.RC_E_STATE
+        else:
+            ix[j, m] = N + 5
+            code = rc.RC_E_INDEX
+    with pytest.raises(rc.RcError) as e:
+        g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, st, oc, pay, ix, n, K)
+    assert e.value.code == code
+    assert f"step {j}," in str(e.value), str(e.value)
+
+
+@pytest.mark.parametrize("kernel", ["gpair", "link", "owned", "split", "tma", "plain"])
 @pytest.mark.parametrize("SB,P", [(16, 32), (16, 64), (64, 128), (64, 32)])
 @pytest.mark.parametrize("K,N,identity", [(1032, 5000, False), (4104, 9001, False), (4104, 4200, False),
                                           (2048, 2048, True), (65536, 70000, False), (65536, 1 << 20, False)])
@@ -285,11 +341,13 @@ def test_persistent_grid_kernels(g, rc, monkeypatch, kernel, SB, P, K, N, identi
     multiple of 8), TMA-fed and plain, on member counts that do not split
     evenly over SMs, with sessions recurring from step to step (N near K);
     "link" is the grid chain split by links (the default for explicit
-    sessions), the others turn it off."""
+    sessions), "gpair" the grid chain keying two steps per barrier (opt-in),
+    the others turn both off."""
     monkeypatch.setenv("RC_OWNED", "1" if kernel == "owned" else "0")
     monkeypatch.setenv("RC_SPLIT", "1" if kernel == "split" else "0")
     monkeypatch.setenv("RC_NO_TMA", "1" if kernel == "plain" else "0")
     monkeypatch.setenv("RC_NO_GRID_LINK", "0" if kernel == "link" else "1")
+    monkeypatch.setenv("RC_GRID_PAIR", "1" if kernel == "gpair" else "0")
     monkeypatch.setenv("RC_NO_CLUSTER", "1")  # K <= 8192 would otherwise take the cluster kernel
     S = 256 if SB == 64 else 64
     tables, state0, outc, pay, idx = _inputs(50 + K % 11, K, S, SB, P, 3, N=None if identity else N)
@@ -299,13 +357,14 @@ def test_persistent_grid_kernels(g, rc, monkeypatch, kernel, SB, P, K, N, identi
     g.assert_same(got, want, f"grid {kernel} K={K} N={N} SB={SB} P={P}")
 
 
-@pytest.mark.parametrize("kernel", ["link", "owned", "split", "tma", "plain"])
+@pytest.mark.parametrize("kernel", ["gpair", "link", "owned", "split", "tma", "plain"])
 def test_grid_barrier_wait_is_bounded_every_grid_kernel(g, rc, monkeypatch, kernel):
     import torch
     monkeypatch.setenv("RC_OWNED", "1" if kernel == "owned" else "0")
     monkeypatch.setenv("RC_SPLIT", "1" if kernel == "split" else "0")
     monkeypatch.setenv("RC_NO_TMA", "1" if kernel == "plain" else "0")
     monkeypatch.setenv("RC_NO_GRID_LINK", "0" if kernel == "link" else "1")
+    monkeypatch.setenv("RC_GRID_PAIR", "1" if kernel == "gpair" else "0")
     monkeypatch.setenv("RC_NO_CLUSTER", "1")  # K <= 8192 would otherwise take the cluster kernel
     K, S, SB, P, n = 8192, 16, 16, 64, 4
     tables, state0, outc, pay, idx = _inputs(19, K, S, SB, P, 2, N=9000)
