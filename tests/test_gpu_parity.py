@@ -332,6 +332,49 @@ def test_grid_pair_errors_report_the_earlier_step(g, rc, monkeypatch, what):
     assert f"step {j}," in str(e.value), str(e.value)
 
 
+@pytest.mark.parametrize("what", ["state_first", "outcome_linked", "outcome_forward", "index"])
+def test_grid_link_errors_report_their_step(g, rc, monkeypatch, what):
+    """The grid chain split by links keys a linked member from the state its
+    session's previous step publishes: a bad state carried that way is
+    reported at the step it was first met, a bad outcome of a linked member
+    or of one whose session goes on into the next step at its own step, a bad
+    index at its own step; a clean chain right after matches the oracle."""
+    monkeypatch.setenv("RC_NO_CLUSTER", "1")
+    monkeypatch.setenv("RC_GRID_PAIR", "0")
+    monkeypatch.setenv("RC_NO_GRID_LINK", "0")
+    K, S, SB, P, n, N = 4104, 64, 16, 64, 6, 4400
+    tables, state0, outc, pay, idx = _inputs(210, K, S, SB, P, n, N=N)
+    st, oc, ix = state0.copy(), outc.copy(), idx.copy()
+    if what == "state_first":
+        # a session of step 0 that is also in step 1 (its state reaches step 1 published)
+        j = 0
+        m = int(np.flatnonzero(np.isin(idx[0], idx[1]))[0])
+        st[int(idx[0, m]), 0:4] = np.frombuffer(np.uint32(S + 3).tobytes(), np.uint8)
+        code = rc.RC_E_STATE
+    elif what == "outcome_linked":
+        j = 2
+        m = int(np.flatnonzero(np.isin(idx[2], idx[1]))[0])
+        oc[j, m] = 9
+        code = rc.RC_E_STATE
+    elif what == "outcome_forward":
+        j = 2
+        m = int(np.flatnonzero(np.isin(idx[2], idx[3]) & ~np.isin(idx[2], idx[1]))[0])
+        oc[j, m] = 9
+        code = rc.RC_E_STATE
+    else:
+        j = 3
+        m = int(np.flatnonzero(np.isin(idx[3], idx[2]))[0])
+        ix[j, m] = N + 5
+        code = rc.RC_E_INDEX
+    with pytest.raises(rc.RcError) as e:
+        g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, st, oc, pay, ix, n, K)
+    assert e.value.code == code
+    assert f"step {j}," in str(e.value), str(e.value)
+    want = g.run_oracle(tables, state0, outc, pay, idx, n, sel0=1)
+    got = g.run_gpu(rc.RC_MECH_RESIDENT_PERSIST, tables, state0, outc, pay, idx, n, K, sel0=1)
+    g.assert_same(got, want, f"grid link after {what}")
+
+
 @pytest.mark.parametrize("kernel", ["gpair", "link", "owned", "split", "tma", "plain"])
 @pytest.mark.parametrize("SB,P", [(16, 32), (16, 64), (64, 128), (64, 32)])
 @pytest.mark.parametrize("K,N,identity", [(1032, 5000, False), (4104, 9001, False), (4104, 4200, False),
