@@ -326,7 +326,8 @@ def native(args):
         hz = {"resident_persist": horizon(rc.RC_MECH_RESIDENT_PERSIST), "host_rt": horizon(rc.RC_MECH_HOST_RT),
               "resident_cond": horizon(rc.RC_MECH_RESIDENT_COND)}
         floor_probe = {name: rc.rc_launch_floor(ctx, kind, 2000 if kind in (0, 3) else 1000) for name, kind in
-                       (("launch_sync", 0), ("graph_node", 1), ("while_iteration", 2), ("launch_d2h_sync", 3))}
+                       (("launch_sync", 0), ("graph_node", 1), ("while_iteration", 2), ("launch_d2h_sync", 3),
+                        ("grid_barrier_step", 4))}
 
         # end to end through the C ABI: events from pinned host memory, decisions
         # and effects back to pinned host memory, inside the timed region
@@ -437,6 +438,9 @@ def large_k(args, rc, torch, stream, hbm_peak, peak_src, flush, world):
             if r > 0:
                 ms_l.append(ms)
         res[name] = float(np.median(ms_l))
+    # floor of one large-K step: an empty step of a persistent chain over one
+    # CTA per SM, the same grid barrier with no member work
+    barrier_us = rc.rc_launch_floor(ctx, 4, 1000)
     rc.rc_free(ctx)
     ms = res["resident_persist"]
     us_inv = ms * 1000.0 / n
@@ -455,6 +459,8 @@ def large_k(args, rc, torch, stream, hbm_peak, peak_src, flush, world):
                      "algorithmic_bytes_per_invocation": alg, "peak_source": f"{peak_src} hbm_gbs (burst)"},
         "l2": "inputs larger than L2 (64 MiB state + 550 MB event ring + 1 GiB effects) and flushed per chain",
         "us_per_invocation_resident": round(us_inv, 4),
+        "grid_barrier_step_floor_us": round(barrier_us, 4),
+        "x_grid_barrier_floor": round(us_inv / barrier_us, 3),
     }
 
 

@@ -182,7 +182,12 @@ int rc_set_wait_limits(rc_ctx *ctx, uint64_t device_ns, uint64_t host_ns);
  * clock); 1 = empty kernel node in a graph of reps back-to-back nodes (device
  * events); 2 = one iteration of an empty WHILE conditional graph (device
  * events); 3 = empty kernel + 4-byte device-to-host copy + synchronise (host
- * clock).  *us_out receives microseconds per unit. */
+ * clock); 4 = one empty step of a persistent chain over one CTA per SM (reps
+ * steps in one cooperative launch, each one grid barrier as the large-K
+ * chain keys it; device events), the floor of a large-K step.  *us_out
+ * receives microseconds per unit.  Kind 4 synchronises and returns
+ * RC_E_TIMEOUT if a barrier wait ran out; other kinds return RC_E_INVAL for
+ * an unknown kind. */
 int rc_launch_floor(rc_ctx *ctx, int kind, uint32_t reps, double *us_out);
 
 /* Device time of the last rc_chain's mechanism work, from CUDA events the

@@ -979,6 +979,28 @@ int rc_launch_floor(rc_ctx *c, int kind, uint32_t reps, double *us_out) {
         *us_out = ns / reps / 1000.0;
         return RC_OK;
     }
+    if (kind == 4) {
+        cudaEvent_t e0 = nullptr, e1 = nullptr;
+        cudaError_t e = cudaEventCreate(&e0);
+        if (e == cudaSuccess) e = cudaEventCreate(&e1);
+        float ms = 0.f;
+        for (int it = 0; it < 3 && e == cudaSuccess; ++it) {  // two warm-ups, then the timed launch
+            e = cudaMemsetAsync(c->dev->slot, 0, sizeof(c->dev->slot), c->stream);
+            if (e == cudaSuccess) e = cudaMemsetAsync(&c->dev->abort, 0, sizeof(uint32_t), c->stream);
+            if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+            if (e == cudaSuccess) e = cudaEventRecord(e0, c->stream);
+            if (e == cudaSuccess) e = rc::launch_grid_barrier_floor(c->dev, reps, c->stream);
+            if (e == cudaSuccess) e = cudaEventRecord(e1, c->stream);
+            if (e == cudaSuccess) e = cudaEventSynchronize(e1);
+            if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, e0, e1);
+        }
+        if (e0) cudaEventDestroy(e0);
+        if (e1) cudaEventDestroy(e1);
+        if (e != cudaSuccess) return cuda_fail(c, e, "grid-barrier floor probe");
+        if ((rc = finish(c)) != RC_OK) return rc;  // a barrier wait that ran out
+        *us_out = static_cast<double>(ms) * 1000.0 / reps;
+        return RC_OK;
+    }
     if (kind != 1 && kind != 2) return fail(c, RC_E_INVAL, "unknown probe kind %d", kind);
     cudaGraph_t g = nullptr;
     cudaGraphExec_t ge = nullptr;

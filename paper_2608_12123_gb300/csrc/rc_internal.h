@@ -207,5 +207,8 @@ const void *launcher_kernel();
 // Launch-floor probes.
 const void *empty_kernel();
 const void *countdown_kernel();
+// n_steps empty grid-barrier steps over one CTA per SM (cooperative launch);
+// dev->slot and dev->abort must be zero.
+cudaError_t launch_grid_barrier_floor(DevBlock *dev, uint32_t n_steps, cudaStream_t s);
 
 }  // namespace rc

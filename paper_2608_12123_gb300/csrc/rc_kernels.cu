@@ -3978,6 +3978,45 @@ __global__ void k_set_word(uint32_t *p, uint32_t v) { *p = v; }
 
 __global__ void k_empty() {}
 
+// Launch-floor probe of the persistent grid chains: one CTA per SM runs
+// n_steps empty steps, each one grid barrier exactly as the large-K chain
+// keys it (block barrier, release add of (1 << 32 | count) to the step's
+// word, CTA 0 clearing the word two steps back, acquire spin bounded by
+// dev->wait_ns, block barrier), with no member work between barriers.
+__global__ void __launch_bounds__(480, 1) k_grid_barrier_floor(DevBlock *dev, uint32_t n_steps) {
+    __shared__ uint32_t s_stop;
+    const uint32_t G = gridDim.x;
+    const uint64_t limit = dev->wait_ns;
+    if (threadIdx.x == 0) s_stop = 0;
+    __syncthreads();
+    for (uint32_t n = 0; n < n_steps; ++n) {
+        if (threadIdx.x == 0) {
+            unsigned long long *word = &dev->slot[n % 3u];
+            if (blockIdx.x == 0) dev->slot[(n + 1u) % 3u] = 0ull;
+            red_release_add_u64(word, (1ull << 32) | (blockIdx.x & 1u));
+            uint64_t t0 = 0;
+            uint32_t spins = 0;
+            for (;;) {
+                if ((ld_acquire_u64(word) >> 32) >= G) break;
+                if ((++spins & 63u) == 0u) {
+                    if (ld_volatile_u32(&dev->abort) != 0u) {
+                        s_stop = 1;
+                        break;
+                    }
+                    if (timed_out(t0, limit)) {
+                        latch_error(dev, DEV_E_TIMEOUT, n, blockIdx.x);
+                        atomicExch(&dev->abort, 1u);
+                        s_stop = 1;
+                        break;
+                    }
+                }
+            }
+        }
+        __syncthreads();
+        if (s_stop != 0u) break;
+    }
+}
+
 __global__ void k_countdown(DevBlock *dev, cudaGraphConditionalHandle h) {
     const uint32_t left = dev->countdown - 1u;
     dev->countdown = left;
@@ -4860,6 +4899,18 @@ cudaError_t launch_set_word(uint32_t *p, uint32_t v, cudaStream_t s) {
 const void *launcher_kernel() { return reinterpret_cast<const void *>(&k_launch_child); }
 const void *empty_kernel() { return reinterpret_cast<const void *>(&k_empty); }
 const void *countdown_kernel() { return reinterpret_cast<const void *>(&k_countdown); }
+
+cudaError_t launch_grid_barrier_floor(DevBlock *dev, uint32_t n_steps, cudaStream_t s) {
+    int d = 0, sms = 0, per_sm = 0;
+    cudaError_t e = cudaGetDevice(&d);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, d);
+    const void *fn = reinterpret_cast<const void *>(&k_grid_barrier_floor);
+    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, 480, 0);
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) return cudaErrorCooperativeLaunchTooLarge;
+    void *args[] = {&dev, &n_steps};
+    return cudaLaunchCooperativeKernel(fn, dim3(sms), dim3(480), args, 0, s);
+}
 
 // ---------------------------------------------------------------------------
 // Allocation-free cohort step (rc_cohort_step_noalloc in include/rc.h).

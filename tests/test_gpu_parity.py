@@ -248,13 +248,28 @@ def test_grid_barrier_wait_is_bounded(g, rc, monkeypatch):
 
 
 def test_launch_floor_probes_run(g, rc):
+    """Every launch-floor probe returns a positive time (kind 4: empty grid
+    steps over one CTA per SM, each wait bounded at 2 ms); an unknown kind is
+    refused; the context then still runs a chain bit-exactly."""
     import torch
-    tables, state0, *_ = _inputs(1, 32, 16, 16, 32, 1)
-    ctx = rc.rc_init(16, tables, 16, 32, 32, 32, torch.cuda.current_stream())
+    K, S, SB, P, n = 32, 16, 16, 32, 6
+    tables, state0, outc, pay, _ = _inputs(1, K, S, SB, P, n)
+    ctx = rc.rc_init(S, tables, SB, P, K, K, torch.cuda.current_stream())
     try:
-        for kind in (0, 1, 2, 3):
+        rc.rc_set_wait_limits(ctx, 2_000_000, 30_000_000_000)
+        for kind in (0, 1, 2, 3, 4):
             us = rc.rc_launch_floor(ctx, kind, 200)
             assert 0.0 < us < 1000.0
+        with pytest.raises(rc.RcError) as e:
+            rc.rc_launch_floor(ctx, 5, 10)
+        assert e.value.code == rc.RC_E_INVAL
+        want = g.run_oracle(tables, state0, outc, pay, None, n)
+        state = g.dev(state0.copy())
+        ev = rc.make_events(g.dev(outc), g.dev(pay), None, payload_bytes=P, n_sets=n)
+        dec = torch.zeros(n, dtype=torch.int32, device="cuda")
+        rc.rc_chain(ctx, n, rc.RC_MECH_RESIDENT_PERSIST, state, ev, K, dec)
+        assert np.array_equal(g.host(dec, np.uint32), want["decisions"])
+        assert np.array_equal(g.host(state, np.uint8).reshape(state0.shape), want["state"])
     finally:
         rc.rc_free(ctx)
 
