@@ -60,6 +60,8 @@ def parse_args():
     p.add_argument("--tiny-only", action="store_true",
                    help="run only the tiny chain's resident leg (profiling)")
     p.add_argument("--large-k-steps", type=int, default=1000)
+    p.add_argument("--large-k-trace", action="store_true",
+                   help="instead of the bench line: phase clocks of one traced large-K chain (profiling)")
     p.add_argument("--only-resident", action="store_true",
                    help="time only the resident chain of the headline workload (profiling)")
     p.add_argument("--no-flush", action="store_true", help="do not allocate or write the L2 flush buffer (profiling)")
@@ -258,6 +260,9 @@ def native(args):
 
     if args.tiny_only:
         print(json.dumps(tiny_chain(rc, torch, stream, mechanisms=("resident_persist",))))
+        return None
+    if args.large_k_trace:
+        print(json.dumps(large_k_trace(rc, torch, stream)))
         return None
     if not args.large_k_only:
         w = make_config2()
@@ -462,6 +467,53 @@ def large_k(args, rc, torch, stream, hbm_peak, peak_src, flush, world):
         "grid_barrier_step_floor_us": round(barrier_us, 4),
         "x_grid_barrier_floor": round(us_inv / barrier_us, 3),
     }
+
+
+def large_k_trace(rc, torch, stream, n=200):
+    """Phase clocks (clock64, rc_set_trace) of one resident chain of n steps of
+    the large-cohort workload: medians over the steady steps of the cycles
+    each phase of k_chain_grid_link takes, for its first and its last CTA.
+    Control thread: release add, effect store and event issue, spin for the
+    slowest CTA.  Member thread 0: region A (linked members gathered and
+    keyed; then every member transitioned and stored) and region B (the next
+    step's unlinked members gathered and keyed)."""
+    n_sets = C4["n_sets"]
+    w = make_config4(n_sets)
+    K, S, SB, P, N = C4["K"], C4["S"], C4["state_bytes"], C4["payload_bytes"], C4["N"]
+    ctx = rc.rc_init(S, w["tables"], SB, P, K, N, stream)
+    state = torch.from_numpy(w["state0"]).cuda()
+    ev = rc.make_events(torch.from_numpy(w["outcome"].view(np.int32)).cuda(), torch.from_numpy(w["payload"]).cuda(),
+                        torch.from_numpy(w["idx"].view(np.int32)).cuda(), payload_bytes=P, n_sets=n_sets)
+    dec = torch.zeros(n, dtype=torch.int32, device="cuda")
+    eff = torch.empty(n * K * 16, dtype=torch.uint8, device="cuda")
+    for _ in range(3):
+        rc.rc_chain(ctx, n, rc.RC_MECH_RESIDENT_PERSIST, state, ev, K, dec, eff, None)
+    untraced_ms, _ = rc.rc_last_chain_stats(ctx)
+    tr = torch.zeros(2 * n * 8, dtype=torch.int64, device="cuda")
+    rc.rc_set_trace(ctx, tr)
+    rc.rc_chain(ctx, n, rc.RC_MECH_RESIDENT_PERSIST, state, ev, K, dec, eff, None)
+    torch.cuda.synchronize()
+    rc.rc_set_trace(ctx, None)
+    rc.rc_free(ctx)
+    t = tr.cpu().numpy().reshape(2, n, 8).astype(np.int64)
+    lo, hi = n // 10, n - 2  # steady steps
+    out = {"workload": "large cohort (K=65,536, N=1,048,576, 64-byte state, 128-byte payload), "
+                       f"one resident chain of {n} steps, SM cycles (clock64), medians over steps {lo}..{hi - 1}",
+           "kernel": "k_chain_grid_link<64,128>",
+           "us_per_step_untraced": round(untraced_ms * 1000.0 / n, 4)}
+    for b, name in ((0, "first_cta"), (1, "last_cta")):
+        x = t[b, lo:hi]
+        med = lambda v: float(np.median(v))  # noqa: E731
+        out[name] = {
+            "ctl_release_add": med(x[:, 1] - x[:, 0]),
+            "ctl_effects_and_event_issue": med(x[:, 2] - x[:, 1]),
+            "ctl_spin": med(x[:, 3] - x[:, 2]),
+            "members_A_linked_gather_and_key": med(x[:, 5] - x[:, 4]),
+            "members_A_transition_and_stores": med(x[:, 6] - x[:, 5]),
+            "members_B_next_unlinked_gather_and_key": med(x[:, 7] - x[:, 6]),
+            "step_period": med(np.diff(t[b, lo:hi + 1, 4])),
+        }
+    return out
 
 
 def tiny_chain(rc, torch, stream, mechanisms=("resident_persist", "resident_cond", "host_rt")):
