@@ -226,6 +226,45 @@ def test_chain_decision_selects_next_body():
     assert effect_fields(out["effects"][0, 0])[2] == T_B[0][0] | (1 << 24)
 
 
+def test_two_sessions_three_steps_worked_by_hand():
+    """Two sessions over three chained steps of two members (S = 4, one
+    payload word each, explicit session order changing between steps).
+    Trajectory worked out by hand from T_A / T_B; each payload word is built
+    from the hand-derived pre-step state so that the member's route key is a
+    chosen published SplitMix64 output (seed 0, output k = mix(k * gamma)):
+    the key matches only if the oracle enters the step with exactly that
+    state, outcome and session.
+
+    step 0, body A: s0 x=1 o=3 -> T_A[1][3]=2, key out 1 (odd); s1 x=3 o=1 ->
+      T_A[3][1]=0, key out 3 (odd); 2 odd of 2 > 1 -> d0 = 1.
+    step 1, body B: s1 x=0 o=2 -> T_B[0][2]=1 (A: 2), key out 2 (even); s0
+      x=2 o=6 -> T_B[2][6]=2 (A: 1), key out 1 (odd); 1 odd -> d1 = 0.
+    step 2, body A: s0 x=2 o=1 -> T_A[2][1]=1 (B: 3), key out 4 (even); s1
+      x=1 o=4 -> T_A[1][4]=0 (B: 3), key out 3 (odd); 1 odd -> d2 = 0."""
+    idx = np.array([[0, 1], [1, 0], [0, 1]], np.uint32)
+    outc = np.array([[3, 1], [2, 6], [1, 4]], np.uint32)
+    pre_x = [[1, 3], [0, 2], [2, 1]]   # hand-derived state entering each step
+    out_k = [[1, 3], [2, 1], [4, 3]]   # published output chosen for each key
+    post_x = [[2, 0], [1, 2], [1, 0]]  # hand-derived next states
+    sels = [0, 1, 0]
+    words = [[oracle.mix64((pre_x[j][m] | int(outc[j, m]) << 32) ^ G) ^ (out_k[j][m] * G & M)
+              for m in range(2)] for j in range(3)]
+    pay = np.frombuffer(b"".join(le(w) for row in words for w in row), np.uint8).reshape(3, 2, 8).copy()
+    state = np.stack([rec16(1, 0, 0), rec16(3, 0, 0)])
+    out = oracle.chain(TABLES, state, outc, pay, idx, n_steps=3, sel0=0)
+    assert [int(d) for d in out["decisions"]] == [1, 0, 0]
+    for j in range(3):
+        for m in range(2):
+            rk, s, packed = effect_fields(out["effects"][j, m])
+            assert rk == K0[out_k[j][m] - 1], (j, m)
+            assert s == idx[j, m]
+            assert packed == post_x[j][m] | (int(outc[j, m]) << 16) | (sels[j] << 24), (j, m)
+            x, step, _ = fields16(out["state_log"][j, m])
+            assert (x, step) == (post_x[j][m], j + 1), (j, m)
+    assert fields16(state[0])[:2] == (1, 3) and fields16(state[1])[:2] == (0, 3)
+    assert out["sel"] == 0
+
+
 def _random_chain(K=32, S=16, P=32, n_steps=200, SB=16, N=None, n_sets=7, cfg=91):
     tables = wl.make_tables(S, wl.stream_seed(cfg, wl.Purpose.TABLE))
     Nn = K if N is None else N
