@@ -201,6 +201,29 @@ def test_former_worked_fixture():
     assert mem.size == fx["A_count"]
 
 
+def test_gap_closure_and_online_ratio_worked_by_hand():
+    """G (Eq. 7) and R_A (Eq. 9) on counts worked out by hand (K = 2,
+    delta = 10, windows from origin 0).  Route 0 is the former fixture's
+    events: windows [0,10) and [30,40) hold 3 and 2 -> F = 5; blocks {0,5,8}
+    and one of {20,30} / {30,31} (a block of three would span 11) -> P = 5;
+    every event shares some interval with another -> U = 6; the former
+    launches {0,8} and {20,30} -> A = 4.  Route 1 is one pair {9,10} split by
+    the window boundary: F = 0, P = U = A = 2.  Together F, P, U, A = 5, 7,
+    8, 6: G = (7 - 5) / (8 - 5) = 2/3, R_A = (6 - 5) / (7 - 5) = 1/2.  Route 0
+    alone has P = F: G = 0, R_A undefined."""
+    t = np.array([0, 5, 8, 9, 10, 20, 30, 31], np.int64)
+    r = np.array([0, 0, 0, 1, 1, 0, 0, 0], np.uint32)
+    s = np.array([1, 1, 2, 6, 7, 3, 4, 5], np.uint32)
+    sh = oracle.shares(t, r, s, 2, 2, 10)
+    assert sh["counts"] == dict(F=5, P=7, U=8, A=6)
+    assert sh["G"] == pytest.approx(2 / 3, abs=1e-15)
+    assert sh["R_A"] == pytest.approx(0.5, abs=1e-15)
+    only0 = r == 0
+    sh0 = oracle.shares(t[only0], r[only0], s[only0], 1, 2, 10)
+    assert sh0["counts"] == dict(F=5, P=5, U=6, A=4)
+    assert sh0["G"] == 0.0 and sh0["R_A"] is None
+
+
 def _check_former(t, r, s, K, delta, mem, tau, cr):
     used = mem.reshape(-1)
     assert len(np.unique(used)) == len(used)                 # each event at most once
